@@ -1,0 +1,437 @@
+"""Benchmark of the MemDecay decode-time eviction loop on GB300.
+
+One step = one pass of the whole hot path over one batch: md_decode_step
+(append + stage-1 paged GQA attention with per-token attention mass) and
+md_evict (stages 2-4: retention priorities, page priorities, budgeted radix
+selection and compaction).  Metric: cached tokens scored + evicted per second
+per decode step (sum over sequences of |K_t| / step time).
+
+Default workload: the largest single-GPU configuration, config 4 (Qwen2.5-3B
+attention geometry, 16 sequences x 131,072 tokens, pages of 32, budget 5%,
+w = 1), at its full-trace step: the first decode step after the prefill,
+attending over the whole trace (77 GB of K/V) and evicting down to budget.
+The device state is restored (untimed) before every timed step, so every
+step does that full work; `--phase steady` times continuing steps instead.
+
+`--impl reference` times the fp64 CPU oracle on the host cores on a bounded
+sample of the same workload (the paper ships no code; the oracle is the
+reference implementation of its equations).
+"""
+from __future__ import annotations
+
+import argparse
+import copy
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "cached tokens scored+evicted per second per decode step"
+UNIT = "tokens/s"
+SPEC_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--w", type=float, default=1.0, help="attention weight (config 4 sweeps 0/0.5/1/4)")
+    ap.add_argument("--phase", default="full", choices=["full", "steady"])
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def source_hash():
+    h = hashlib.sha256()
+    with open(os.path.join(ROOT, "paper_2607_10582_gb300", "csrc", "md_attn.cu"), "rb") as f:
+        h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic_per_token():
+    """DRAM bytes per cached token per layer of the attention kernel, from the
+    committed ncu summary, if it was taken on the current kernel source."""
+    p = os.path.join(ROOT, "profiles", "attn_mass_kernel_traffic.txt")
+    if not os.path.exists(p):
+        return None
+    vals = {}
+    with open(p) as f:
+        for line in f:
+            if ":" in line and not line.startswith("#"):
+                k, v = line.split(":", 1)
+                vals[k.strip()] = v.strip()
+    if vals.get("kernel_source_sha256_16") != source_hash():
+        return None
+    try:
+        return float(vals["dram_bytes_per_token_layer"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi samples during the timed region (the GPU's clocks and
+    throttle reasons are read, never set)."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], 0.0, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = max(mx, float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------- native ----
+def run_native(args, rank, world, local_rank):
+    import torch
+    import paper_2607_10582_gb300 as md
+    from paper_2607_10582_gb300 import build as mdbuild
+    import synth
+
+    mdbuild.build()
+    synth.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.current_stream(dev)
+    over = {"attn_weight": args.w} if args.config == 4 else {}
+    w = synth.make_workload(args.config, seed=args.seed + rank, **over)
+    B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
+    cache = md.Cache(L, Hq, Hkv, ps, B, w.max_pages_per_seq(), w.num_phys_pages(),
+                     rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
+                     score_mode=w.score_mode, page_reduce=w.page_reduce, keep_token_prio=0)
+    for r in range(7):
+        cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    lib = synth.lib()
+    kap = None
+    nmax = max(w.n0(b) for b in range(B))
+    kbuf = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
+    vbuf = torch.empty_like(kbuf)
+    for b in range(B):
+        n = w.n0(b)
+        reg_d = torch.from_numpy(w.regions[b]).to(dev)
+        assert lib.synth_fill_kv_dev(w.seed, int(w.structured), kap, b, L, Hkv, D, 0, n, reg_d.data_ptr(),
+                                     kbuf.data_ptr(), vbuf.data_ptr(), stream.cuda_stream) == 0
+        cache.append_tokens(b, w.regions[b], kbuf.data_ptr(), vbuf.data_ptr(), w.insert_steps[b])
+    del kbuf, vbuf
+    torch.cuda.synchronize()
+
+    # per-step inputs, resident in HBM
+    q = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((B, L, Hkv, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    out = torch.empty_like(q)
+    pos_d = torch.tensor([w.n0(b) for b in range(B)], dtype=torch.int32, device=dev)
+    regs = [w.decode_region] * B
+    reg_d = torch.tensor(regs, dtype=torch.uint8, device=dev)
+    assert lib.synth_fill_q_dev(w.seed, int(w.structured), kap, B, L, Hq, Hq // Hkv, D, 1, q.data_ptr(),
+                                stream.cuda_stream) == 0
+    assert lib.synth_fill_step_kv_dev(w.seed, int(w.structured), kap, B, L, Hkv, D, pos_d.data_ptr(),
+                                      reg_d.data_ptr(), kn.data_ptr(), vn.data_ptr(), stream.cuda_stream) == 0
+    torch.cuda.synchronize()
+    budgets = list(w.budget_pages)
+
+    def one_step():
+        cache.decode_step(B, q, kn, vn, regs, out)
+        # observation every window_k steps (k = 1 for configs 0-2 and 4)
+        if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
+            cache.evict(budgets)
+
+    if args.phase == "steady":
+        one_step()
+        if cache.query(md.MD_QUERY_WINDOW) > 0:
+            cache.evict(budgets)
+        torch.cuda.synchronize()
+    saved = cache.save_state()
+    tokens_step = sum(cache.query(md.MD_QUERY_TOKENS, b) + 1 for b in range(B))
+    restore = args.phase == "full"
+
+    for _ in range(args.warmup):
+        if restore:
+            cache.load_state(saved)
+        one_step()
+    torch.cuda.synchronize()
+    assert cache.sync() == md.MD_OK
+
+    # ---- timed region: K steps, CUDA events on the launching stream ----
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    tok_per_step = []
+    clocks = ClockSampler(local_rank) if not args.no_clocks else None
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    cache.profile_enable(True)
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        if restore:
+            cache.load_state(saved)
+        tok_per_step.append(sum(cache.query(md.MD_QUERY_TOKENS, b) + 1 for b in range(B)))
+        starts[i].record(stream)
+        one_step()
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop() if clocks else None
+    prof = cache.profile_read()
+    cache.profile_enable(False)
+    assert cache.sync() == md.MD_OK
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_ms = float(sum(step_ms))
+    launches = sum(n for _, n in prof.values())
+    attn_ms, attn_n = prof["attention"]
+
+    # ---- end to end through the C ABI with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        qh = q.cpu().pin_memory()
+        knh = kn.cpu().pin_memory()
+        vnh = vn.cpu().pin_memory()
+        outh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+        e_ms = []
+        for i in range(args.warmup + args.steps):
+            if restore:
+                cache.load_state(saved)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            q.copy_(qh, non_blocking=True)
+            kn.copy_(knh, non_blocking=True)
+            vn.copy_(vnh, non_blocking=True)
+            one_step()
+            outh.copy_(out, non_blocking=True)
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                e_ms.append((time.perf_counter() - t0) * 1e3)
+        h2d = (qh.numel() + knh.numel() + vnh.numel()) * 2 + B
+        d2h = outh.numel() * 2
+        e2e = {"ms_per_step": float(np.mean(e_ms)), "tokens_per_step": tok_per_step[0],
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+    return dict(w=w, step_ms=step_ms, total_ms=total_ms, wall_s=wall, tokens=tok_per_step,
+                prof=prof, launches=launches, attn_ms=attn_ms, attn_n=attn_n, clocks=clk, e2e=e2e,
+                kv_bytes_per_token=L * Hkv * 2 * D * 2)
+
+
+# ------------------------------------------------------------ reference ----
+def oracle_sample(w, layers: int, seq: int = 0):
+    """Build the oracle for one sequence of workload w, keeping `layers` of its
+    L layers (the attention work is linear in L), prefilled (untimed)."""
+    import oracle.memdecay_oracle as om
+    import synth
+    n = w.n0(seq)
+    cfg = om.OracleConfig(layers, w.Hq, w.Hkv, w.D, w.page_size, 1, w.max_pages_per_seq(),
+                          w.pages0(seq) + w.steps // w.page_size + 2, rho=w.rho, gamma=w.gamma,
+                          tau_scale=w.tau_scale, attn_weight=w.attn_weight, score_mode=w.score_mode,
+                          page_reduce=w.page_reduce)
+    o = om.Oracle(cfg)
+    for r in range(7):
+        o.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    k, v = synth.kv_host(w.seed, seq, layers, w.Hkv, 0, n, w.regions[seq], w.structured)
+    o.append_tokens(0, w.regions[seq], k, v, w.insert_steps[seq])
+    q = synth.q_host(w.seed, 1, layers, w.Hq, w.Hkv, 1, w.structured)
+    kn, vn = synth.step_kv_host(w.seed, [n], [w.decode_region], layers, w.Hkv, w.structured)
+    return o, (q, kn, vn)
+
+
+def time_oracle_step(o, inputs, w, layers):
+    """One oracle step on the sample; returns the estimated seconds of the
+    whole workload's step (all L layers, all B sequences)."""
+    q, kn, vn = inputs
+    t0 = time.perf_counter()
+    o.decode_step(1, q, kn, vn, [w.decode_region])
+    t1 = time.perf_counter()
+    o.evict(1, [w.budget_pages[0]])
+    t2 = time.perf_counter()
+    per_seq = (t1 - t0) * (w.L / layers) + (t2 - t1)
+    return per_seq * w.B, (t1 - t0), (t2 - t1)
+
+
+def cpu_cores_used():
+    return 1
+
+
+def run_reference(args):
+    import synth
+    over = {"attn_weight": args.w} if args.config == 4 else {}
+    w = synth.make_workload(args.config, seed=args.seed, **over)
+    layers = 1
+    o0, inputs = oracle_sample(w, layers)
+    tokens_step = sum(w.n0(b) + 1 for b in range(w.B))
+    est = []
+    for i in range(args.warmup + args.steps):
+        o = copy.deepcopy(o0)
+        s, _, _ = time_oracle_step(o, inputs, w, layers)
+        if i >= args.warmup:
+            est.append(s)
+    sec = float(np.mean(est))
+    value = tokens_step / sec
+    sample = (f"sequence 0 of {w.B}, {layers} of {w.L} layers, full trace ({w.n0(0)} tokens): "
+              f"attention time x{w.L // layers} layers, + scoring/eviction, x{w.B} sequences")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(w, args),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores_used(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(w, args):
+    return {"workload": w.name, "batch": w.B, "tokens_per_seq": w.n0(0), "layers": w.L,
+            "q_heads": w.Hq, "kv_heads": w.Hkv, "head_dim": w.D, "page_size": w.page_size,
+            "budget_pages": w.budget_pages[0], "attn_weight": w.attn_weight, "window_k": w.window_k,
+            "score_mode": "paper additive (Eq. 4)" if w.score_mode == 0 else "multiplicative",
+            "phase": "full-trace step (state restored before each step)" if args.phase == "full"
+            else "steady state",
+            "l2": "no flush: inputs larger than L2 (K/V read per step >> 129 MB)",
+            "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed}
+
+
+# ------------------------------------------------------------------ main ----
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args)
+        return
+    import torch
+    if world > 1:
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    r = run_native(args, rank, world, local_rank)
+    w = r["w"]
+    total_ms = r["total_ms"]
+    tokens = float(np.mean(r["tokens"]))
+    if world > 1:
+        t = torch.tensor([total_ms, tokens * args.steps], dtype=torch.float64, device="cuda")
+        mx = t.clone()
+        torch.distributed.all_reduce(mx[:1], op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.all_reduce(t[1:], op=torch.distributed.ReduceOp.SUM)
+        total_ms = float(mx[0])
+        all_tokens = float(t[1])
+    else:
+        all_tokens = tokens * args.steps
+    if rank != 0:
+        torch.distributed.destroy_process_group()
+        return
+    ms_per_step = total_ms / args.steps
+    value = all_tokens / (total_ms / 1e3)
+    peak, peak_kind = peaks()
+    # dominant kernel: stage-1 attention.  Algorithmic bytes per launch = the
+    # K and V rows of every cached token in every layer, plus Q and O.
+    kv_bytes = tokens * r["kv_bytes_per_token"]
+    qo_bytes = 2 * w.B * w.L * w.Hq * w.D * 2
+    attn_bytes = kv_bytes + qo_bytes
+    attn_avg_s = r["attn_ms"] / max(1, r["attn_n"]) / 1e3
+    achieved = attn_bytes / attn_avg_s / 1e9
+    tpt = ncu_traffic_per_token()
+    traffic = None if tpt is None else tpt * tokens * w.L
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload_config(w, args),
+        "roofline": {"bound": "hbm", "kernel": "attn_mass_kernel (stage 1)", "achieved": achieved,
+                     "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{peak_kind} copy",
+                     "traffic": traffic, "algorithmic_bytes": attn_bytes,
+                     "frac_of_8TBps_spec": achieved / SPEC_HBM_GBS},
+        "step_hbm_fraction": {"algorithmic_GBps": attn_bytes / (ms_per_step / 1e3) / 1e9,
+                              "frac_measured": attn_bytes / (ms_per_step / 1e3) / 1e9 / peak,
+                              "frac_of_8TBps_spec": attn_bytes / (ms_per_step / 1e3) / 1e9 / SPEC_HBM_GBS},
+        "stage_ms_per_step": {k: v[0] / args.steps for k, v in r["prof"].items()},
+        "gpu_launches": r["launches"],
+        "clocks": r["clocks"],
+        "wall_s_timed": r["wall_s"],
+    }
+    if r["e2e"]:
+        e = r["e2e"]
+        line["e2e"] = {"value": e["tokens_per_step"] * world / (e["ms_per_step"] / 1e3), "unit": UNIT,
+                       "ms_per_step": e["ms_per_step"], "h2d_bytes_per_step": e["h2d_bytes_per_step"],
+                       "d2h_bytes_per_step": e["d2h_bytes_per_step"]}
+    if not args.no_cpu_baseline and world == 1:
+        o0, inputs = oracle_sample(w, 1)
+        s, t_dec, t_ev = time_oracle_step(o0, inputs, w, 1)
+        line["cpu_baseline"] = {
+            "value": sum(w.n0(b) + 1 for b in range(w.B)) / s, "unit": UNIT, "cores": cpu_cores_used(),
+            "kind": "oracle",
+            "sample": f"sequence 0 of {w.B}, 1 of {w.L} layers, full trace: oracle decode step "
+                      f"{t_dec:.2f} s x{w.L} layers + observation/eviction {t_ev:.2f} s, x{w.B} sequences"}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

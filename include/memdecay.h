@@ -1,0 +1,242 @@
+/* memdecay.h -- C ABI of the GB300 (sm_103a) MemDecay decode-time eviction loop.
+ *
+ * MemDecay ("MemDecay: Region-Aware KV Cache Eviction for Efficient LLM Agent
+ * Inference", arXiv 2607.10582) keeps, for every cached token i of a paged KV
+ * cache, a region label r(i), an attention importance a_i and a decay clock
+ * t_ref_i.  At every observation step (Algorithm 1) it updates a_i with an
+ * EWMA of the attention mass the token received (Eq. 2), restarts the clock of
+ * tokens attended above a threshold (Eq. 3), scores every token with its
+ * region's decayed base priority plus its weighted importance (Eq. 4), reduces
+ * token scores to page scores (Eq. 5) and, when the cache holds more pages than
+ * the budget, evicts the lowest-scoring non-pinned pages (Sec. III-D).
+ *
+ * This library implements that loop on one GPU, in four stages run by
+ * md_decode_step and md_evict:
+ *   1. paged GQA decode attention that also produces each cached token's
+ *      attention mass (Sec. III-C, observation of Abar_i);
+ *   2. per-token retention priority (Eqs. 2-4);
+ *   3. token -> page priority (Eq. 5, pinning protects whole pages, Sec. IV-A);
+ *   4. budgeted selection of the lowest-priority pages (radix select) and
+ *      compaction of the block table and free list (Sec. III-D, Algorithm 1).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Memory: the library allocates no device memory.  The caller passes one
+ *   device workspace (md_config.workspace) of md_workspace_size() bytes, which
+ *   holds the KV page pool and all per-token / per-page state.  Device
+ *   pointers passed to calls are borrowed for the duration of the call's GPU
+ *   work only; K/V are copied into the pool.
+ * - Streams: every call enqueues its GPU work on md_config.stream (a
+ *   cudaStream_t) and returns without synchronising, except where stated.
+ * - Host mirror: sequence token/page counts, the free-stack top and the step
+ *   counter are tracked exactly on the host, so argument and capacity errors
+ *   are returned synchronously, before anything is launched, and nothing is
+ *   changed when a call fails.
+ * - Device errors (an exchange wait that timed out) are recorded in a sticky
+ *   device status word, read by md_sync(); after one, the handle refuses
+ *   further work (MD_ERR_STATE) and must be destroyed.  No kernel traps.
+ * - Threading: a handle is used from one host thread and one stream.
+ * - Layouts are row-major; bf16 tensors are passed as raw 16-bit patterns.
+ */
+#ifndef MEMDECAY_H
+#define MEMDECAY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct md_ctx md_ctx; /* opaque, host-owned */
+
+typedef enum {
+  MD_OK = 0,
+  MD_WARN_OVER_BUDGET = 1,     /* pinned pages alone exceed a budget: every
+                                  evictable page was evicted, state is valid */
+  MD_ERR_INVALID_ARG = -1,
+  MD_ERR_CAPACITY = -2,        /* block table row or page pool would overflow */
+  MD_ERR_WORKSPACE = -3,       /* workspace missing, misaligned or too small */
+  MD_ERR_CUDA = -4,            /* a CUDA runtime call failed */
+  MD_ERR_DEVICE_TIMEOUT = -5,  /* a bounded device-side wait ran out */
+  MD_ERR_STATE = -6            /* call not valid in the handle's state */
+} md_status;
+
+/* Region labels, in the order Sec. III-A lists them. */
+enum {
+  MD_REGION_SYSTEM = 0,
+  MD_REGION_PLAN = 1,
+  MD_REGION_USER = 2,
+  MD_REGION_TOOL_IN = 3,
+  MD_REGION_TOOL_OUT = 4,
+  MD_REGION_RETRIEVAL = 5,
+  MD_REGION_SCRATCHPAD = 6,
+  MD_NUM_REGIONS = 7
+};
+
+#define MD_MAX_BATCH 256          /* sequences per handle                     */
+#define MD_HEAD_DIM 128           /* the only supported head dimension        */
+#define MD_MAX_GROUP 8            /* query heads per KV head (GQA group)      */
+#define MD_MAX_CHUNKS 64          /* attention splits per (seq, layer, head)  */
+#define MD_MAX_CHUNK_TOKENS 4096  /* tokens per attention split               */
+
+typedef struct {
+  /* Geometry: L layers, Hq query heads, Hkv KV heads (Hq / Hkv <= 8), head_dim
+   * must be 128, page_size 16 or 32 tokens (Sec. III-D, fixed-size pages). */
+  int num_layers, num_q_heads, num_kv_heads, head_dim, page_size;
+  /* Capacity: sequences, block-table width (pages per sequence, at most
+   * MD_MAX_CHUNKS * MD_MAX_CHUNK_TOKENS / page_size), pages in the pool. */
+  int max_batch, max_pages_per_seq, num_phys_pages;
+  /* Policy (Sec. IV-A uses rho 0.9, gamma = 1 - rho, tau = 2 / |K_t|):
+   *   a_i <- rho a_i + gamma Abar_i                           (Eq. 2)
+   *   refresh when Abar_i >= tau_scale / |K_t|                 (Eq. 3)
+   *   score_mode 0: s_i = b_r 2^(-dt/h_r) + attn_weight a_i    (Eq. 4)
+   *   score_mode 1: s_i = (b_r + attn_weight a_i) 2^(-dt/h_r)
+   *   page_reduce 0: S_p = mean over the page's tokens (Eq. 5); 1: max. */
+  float rho, gamma, tau_scale, attn_weight;
+  int score_mode, page_reduce;
+  int keep_token_prio;        /* 1: store s_i per token (md_get_state) */
+  void *workspace;            /* device memory, 256-byte aligned, caller-owned */
+  size_t workspace_bytes;
+  void *stream;               /* cudaStream_t (NULL = legacy default stream) */
+} md_config;
+
+/* Bytes of device workspace md_create needs for cfg (0 if cfg is invalid).
+ * Pure host arithmetic; no CUDA call. */
+size_t md_workspace_size(const md_config *cfg);
+
+/* Validates cfg, lays out the workspace, and enqueues its initialisation
+ * (empty cache, free stack [P-1, ..., 0] so the first page taken is 0).
+ * Region parameters start as b = 0, half-life = +inf, not pinned. */
+md_status md_create(const md_config *cfg, md_ctx **out);
+
+/* Structural prior of one region (Sec. III-B, Table 1): base priority
+ * b_r >= 0 and half-life h_r > 0 in decode steps (lambda_r = ln 2 / h_r,
+ * Eq. 7; h_r = +INFINITY means lambda_r = 0).  pinned != 0 puts the region in
+ * the never-evicted set F (Eq. 1).  The pinned flag can only change while no
+ * sequence holds tokens (MD_ERR_STATE otherwise); b_r and h_r at any time. */
+md_status md_set_region_params(md_ctx *ctx, int region, float base_priority,
+                               float half_life_steps, int pinned);
+
+/* Appends n tokens to sequence seq (the prompt from the orchestrator, Fig. 1
+ * "append KV"; Sec. III-A: every token carries a region label and an
+ * insertion step).
+ *   regions_host      [n] region label per token (host memory)
+ *   insert_steps_host [n] insertion step per token (host), each <= the current
+ *                     step; NULL means the current step for all
+ *   k_dev, v_dev      bf16 [L][Hkv][n][D] (device)
+ * Each token starts with a_i = 0 and t_ref_i = its insertion step.  New pages
+ * are taken from the free stack. */
+md_status md_append_tokens(md_ctx *ctx, int seq, int n_tokens, const uint8_t *regions_host,
+                           const int32_t *insert_steps_host, const void *k_dev,
+                           const void *v_dev);
+
+/* One decode step for sequences [0, batch): advances the step counter t,
+ * appends each sequence's new token (region new_region_host[b], inserted at
+ * t), then runs stage 1: for every layer and query head, attention over every
+ * cached token of the sequence (the new one included; no mask), writing the
+ * output and accumulating each token's attention mass for the observation
+ * window (Sec. III-C).
+ *   q_dev               bf16 [batch][L][Hq][D]    (device)
+ *   k_new_dev, v_new_dev bf16 [batch][L][Hkv][D]  (device)
+ *   new_region_host     [batch]                   (host)
+ *   out_dev             bf16 [batch][L][Hq][D]    (device, written)
+ * All steps of one observation window must use the same batch. */
+md_status md_decode_step(md_ctx *ctx, int batch, const void *q_dev, const void *k_new_dev,
+                         const void *v_new_dev, const uint8_t *new_region_host, void *out_dev);
+
+/* The observation step of Algorithm 1 for sequences [0, batch): stages 2-4.
+ * If decode steps ran since the last call, Abar_i = (attention mass summed
+ * over those k steps, layers and query heads) / (k L Hq), then Eq. 2, Eq. 3
+ * with tau = tau_scale / |K_t| (|K_t| = tokens cached now); if none ran, the
+ * EWMA and the clocks are left as they are.  Then Eq. 4 and Eq. 5 (pinned
+ * pages and each sequence's last page, the one being written, score +inf),
+ * and, for every sequence holding more pages than budget_pages_host[b]
+ * (partial last page included), eviction of the lowest-S_p evictable pages
+ * (ties: lower logical page index first), stable compaction of its block-table
+ * row, and a push of the freed physical ids onto the free stack in
+ * (sequence, logical page) order.
+ *   budget_pages_host [batch]            (host)
+ *   n_evicted_host    [batch] or NULL    (host, written before return: the
+ *                                         counts come from the host mirror)
+ *   evicted_ids_dev   [batch][max_pages_per_seq] or NULL (device, written:
+ *                     freed physical ids in logical order, -1 padded)
+ * Returns MD_WARN_OVER_BUDGET when pinned pages keep a sequence above its
+ * budget. */
+md_status md_evict(md_ctx *ctx, int batch, const int32_t *budget_pages_host,
+                   int32_t *n_evicted_host, int32_t *evicted_ids_dev);
+
+/* Waits for the handle's stream and returns the sticky device status. */
+md_status md_sync(md_ctx *ctx);
+
+md_status md_destroy(md_ctx *ctx);
+
+/* ---- inspection, test and checkpoint support -------------------------- */
+
+enum {
+  MD_STATE_BLOCK_TABLE = 0, /* int32 [max_batch][max_pages_per_seq] physical ids     */
+  MD_STATE_PAGE_SCORE = 1,  /* fp32  [max_batch][max_pages_per_seq] S_p (last evict)  */
+  MD_STATE_TOKEN_PRIO = 2,  /* fp32  [num_phys_pages*page_size] s_i per physical slot */
+  MD_STATE_A = 3,           /* fp32  [slots] a_i                                      */
+  MD_STATE_T_REF = 4,       /* int32 [slots] t_ref_i                                  */
+  MD_STATE_AHAT = 5,        /* fp32  [slots] Abar_i of the last observation           */
+  MD_STATE_FREE = 6,        /* int32 [num_phys_pages] free stack (top: md_query)      */
+  MD_STATE_REGION = 7,      /* uint8 [slots] region label                             */
+  MD_STATE_WINDOW = 8,      /* fp32  [slots] attention mass of folded window steps    */
+  MD_STATE_MASS = 9,        /* fp32  [L*Hkv][slots] mass rows of the last decode step */
+  MD_STATE_POOL = 10        /* bf16  [L][num_phys_pages][Hkv][2][page_size][D] K/V    */
+};
+
+/* Device-to-device copy of one state array into dst_dev (bytes must equal the
+ * array's size), enqueued on the stream. */
+md_status md_get_state(md_ctx *ctx, int what, void *dst_dev, size_t bytes);
+
+/* Overwrites one state array from src_dev (test support: lets a parity test
+ * put the oracle's choice back where floating-point ties allowed the GPU
+ * another valid one).  Only BLOCK_TABLE, FREE, A and T_REF; the caller keeps
+ * the array consistent with the host mirror's counts. */
+md_status md_set_state(md_ctx *ctx, int what, const void *src_dev, size_t bytes);
+
+enum {
+  MD_QUERY_TOKENS = 0,   /* cached tokens of sequence seq            */
+  MD_QUERY_PAGES = 1,    /* resident pages of sequence seq           */
+  MD_QUERY_FREE_TOP = 2, /* free-stack height                        */
+  MD_QUERY_STEP = 3,     /* current decode step t                    */
+  MD_QUERY_WINDOW = 4,   /* decode steps since the last observation  */
+  MD_QUERY_PINNED_PAGES = 5 /* pages of seq holding a pinned token   */
+};
+md_status md_query(const md_ctx *ctx, int what, int seq, int64_t *out);
+
+/* Checkpoint of everything but the page pool's contents: device state into
+ * dst_dev (md_state_bytes() device bytes) and the host mirror into host_blob
+ * (host bytes).  Only between observation windows (MD_ERR_STATE otherwise).
+ * md_load_state restores both; the pool must still hold the saved pages. */
+md_status md_state_bytes(const md_ctx *ctx, size_t *device_bytes, size_t *host_bytes);
+md_status md_save_state(md_ctx *ctx, void *dst_dev, void *host_blob);
+md_status md_load_state(md_ctx *ctx, const void *src_dev, const void *host_blob);
+
+/* Per-stage GPU time, from CUDA events recorded around each launch while
+ * enabled.  Stages: 0 append, 1 attention (stage 1), 2 window fold,
+ * 3 score + page reduce (stages 2-3), 4 select + compact (stage 4).
+ * md_profile_read synchronises the stream and returns, for each stage, the
+ * summed milliseconds and the number of launches since enabling. */
+md_status md_profile_enable(md_ctx *ctx, int enable);
+md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_per_stage,
+                          int n_stages);
+
+/* Test support: bounded waits and injected timeouts.
+ *   MD_DEBUG_SPIN_LIMIT_NS    limit of each device-side wait (default 2e9)
+ *   MD_DEBUG_EXTRA_ARRIVALS   extra arrivals the attention exchange waits for
+ *                             on its next launch (a wait nothing completes;
+ *                             the kernel then reports MD_ERR_DEVICE_TIMEOUT) */
+enum { MD_DEBUG_SPIN_LIMIT_NS = 0, MD_DEBUG_EXTRA_ARRIVALS = 1 };
+md_status md_debug_set(md_ctx *ctx, int key, int64_t value);
+
+/* Text of the last error on this handle ("" if none). */
+const char *md_last_error(const md_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MEMDECAY_H */

@@ -210,13 +210,18 @@ class Oracle:
         self.n_tokens[b] += 1
 
     def append_tokens(self, b: int, regions: np.ndarray, K: np.ndarray, V: np.ndarray,
-                      insert_step: Optional[int] = None) -> None:
-        """Prefill: K, V are bf16 bits [L][Hkv][n][D]; regions [n]."""
-        ts = self.t if insert_step is None else int(insert_step)
-        if ts > self.t:
+                      insert_step=None) -> None:
+        """Prefill: K, V are bf16 bits [L][Hkv][n][D]; regions [n]; insert_step
+        an int, one int per token, or None (the current step)."""
+        n = len(regions)
+        if insert_step is None:
+            steps = np.full(n, self.t, np.int64)
+        else:
+            steps = np.broadcast_to(np.asarray(insert_step, np.int64), (n,))
+        if n and steps.max() > self.t:
             raise ValueError("insert_step after the current step")
-        for i in range(len(regions)):
-            self._append_one(b, int(regions[i]), K[:, :, i, :], V[:, :, i, :], ts)
+        for i in range(n):
+            self._append_one(b, int(regions[i]), K[:, :, i, :], V[:, :, i, :], int(steps[i]))
 
     def slots(self, b: int) -> np.ndarray:
         """Physical slots of sequence b in logical order."""

@@ -1,0 +1,481 @@
+/* Stage 1: paged GQA decode attention that also yields every cached token's
+ * attention mass (Sec. III-C: Abar_i, the attention a token receives averaged
+ * over heads and layers, is what MemDecay observes).
+ *
+ * Work unit: (sequence b, layer l, KV head kvh, chunk j of the sequence's
+ * pages).  The chunks of one (b, l, kvh) item split its pages (flash-decoding
+ * style) so that ~all 152 SMs stream K/V at once.  One persistent cooperative
+ * CTA per SM walks the units c, c+grid, c+2*grid, ...
+ *
+ * Per CTA: warp 0 is the producer.  One elected lane issues, per page, two
+ * TMA tile loads (cp.async.bulk.tensor, 128-byte swizzle, L2 evict_first) of
+ * the page's K and V rows into a ring of shared-memory stages with mbarrier
+ * completion.  Warps 1..NCW consume pages round-robin:
+ *   S^T[16 tokens x 8 heads] = K[16 x 128] . Q^T    (mma.sync m16n8k16 bf16)
+ *   online softmax per head (exp2 domain), raw scores kept in scratch
+ *   O^T[128 x 8] += V^T[128 x 16] . P^T             (P^T via movmatrix.trans)
+ * GQA makes both products real dense tiles: the G <= 8 query heads of one KV
+ * head share every K/V byte read, so K/V are read from HBM once per step.
+ *
+ * Exact mass without re-reading K: a token's mass is sum_h exp(s_hi - m_h)/Z_h
+ * with the item's global (m_h, Z_h).  A unit publishes its partial (m, Z, O)
+ * and bumps the item's arrival counter; one unit later (so nothing waits on
+ * the critical path) the CTA waits, bounded by %globaltimer, for all chunks of
+ * the earlier item, combines the partials (its slice of the output O) and
+ * turns its stored scores into masses, one fp32 row per (layer, KV head)
+ * indexed by physical slot.  All waits are bounded; on expiry the kernel
+ * records MD_ERR_DEVICE_TIMEOUT, raises an abort flag every CTA polls, drains
+ * its in-flight copies and returns.  No float atomics: results are
+ * bit-identical run to run. */
+#include <cuda_bf16.h>
+#include <float.h>
+
+#include "md_internal.h"
+#include "md_ptx.cuh"
+
+namespace md {
+
+template <int PS, int NCW>
+struct AttnShape {
+  static constexpr int NT = PS / 16;                 // 16-token tiles per page
+  static constexpr int HALF_BYTES = 2 * PS * 128;    // 64 columns of K and V rows
+  static constexpr int STAGE_BYTES = 2 * HALF_BYTES; // one page of one (layer, KV head)
+  static constexpr int R = (PS == 16) ? 16 : 8;      // ring stages (128 KiB)
+  static constexpr int RING_BYTES = R * STAGE_BYTES;
+  static constexpr int THREADS = 32 * (NCW + 1);
+  static constexpr int MERGE_FLOATS = NCW * (16 + GP * D);
+  static constexpr int FIN_FLOATS = 16 + MD_MAX_CHUNKS * GP;
+  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * R * 8 + 4 * MERGE_FLOATS +
+                                 4 * FIN_FLOATS + 64;
+};
+
+struct Unit {
+  int b, l, kvh, j, C, p0, p1, X;
+};
+
+__device__ __forceinline__ Unit decode_unit(const AttnParams &p, int u) {
+  int lo = 0, hi = p.n_seqs - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (p.unit_start[mid] <= u) lo = mid; else hi = mid - 1;
+  }
+  Unit un;
+  un.b = lo;
+  un.C = p.chunks[lo];
+  int rem = u - p.unit_start[lo];
+  int item = rem / un.C;
+  un.j = rem - item * un.C;
+  un.l = item / p.Hkv;
+  un.kvh = item - un.l * p.Hkv;
+  int P = p.n_pages[lo];
+  un.p0 = (int)(((long long)un.j * P) / un.C);
+  un.p1 = (int)(((long long)(un.j + 1) * P) / un.C);
+  un.X = (lo * p.L + un.l) * p.Hkv + un.kvh;
+  return un;
+}
+
+__device__ __forceinline__ void raise_status(const AttnParams &p, int code, int diag) {
+  atomicCAS(&p.status[ST_CODE], 0, code);
+  atomicExch(&p.status[ST_DIAG], diag);
+  atomicExch(&p.status[ST_ABORT], 1);
+}
+
+/* Bounded wait on an mbarrier phase; false on abort or timeout. */
+__device__ __noinline__ bool wait_phase(uint32_t bar, uint32_t parity, const AttnParams &p,
+                                        int diag, bool honour_abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = globaltimer();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (honour_abort && ld_volatile(&p.status[ST_ABORT])) return false;
+    if (globaltimer() - t0 > p.spin_limit_ns) {
+      raise_status(p, MD_ERR_DEVICE_TIMEOUT, diag);
+      return false;
+    }
+  }
+}
+
+/* Address of the 16-byte chunk holding (row, d..d+7) of a stage stored as two
+ * 64-column halves of 128-byte rows with the TMA 128-byte swizzle. */
+template <int PS>
+__device__ __forceinline__ uint32_t swz(uint32_t stage, int row, int d) {
+  const int half = d >> 6;
+  const int chunk = (d & 63) >> 3;
+  return stage + half * (2 * PS * 128) + row * 128 + ((chunk ^ (row & 7)) << 4);
+}
+
+template <int PS, int NCW>
+__global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
+    attn_mass_kernel(const __grid_constant__ AttnParams p,
+                     const __grid_constant__ CUtensorMap tmap) {
+  using S = AttnShape<PS, NCW>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t *ring = smem;
+  uint64_t *full = (uint64_t *)(ring + S::RING_BYTES);
+  uint64_t *empty = full + S::R;
+  float *wm = (float *)(empty + S::R);        // [NCW][8] per-warp running max
+  float *wl = wm + NCW * 8;                   // [NCW][8] per-warp running sum
+  float *wO = wl + NCW * 8;                   // [NCW][8][128] per-warp O^T
+  float *fin = wm + S::MERGE_FLOATS;          // [16]: unit max m[8] then 8 spare
+  float *fac = fin + 16;                      // [MD_MAX_CHUNKS][8] combine factors
+  int *flag = (int *)(fac + MD_MAX_CHUNKS * GP);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t ring_u32 = smem_u32(ring);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S::R; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    flag[0] = flag[1] = flag[2] = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  if (warp == 0) {
+    /* ------------------------------------------------------- producer ---- */
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      tma_prefetch_desc(&tmap);
+      int i = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const Unit un = decode_unit(p, u);
+        const int32_t *bt = p.block_table + (size_t)un.b * p.P_max;
+        for (int pg = un.p0; pg < un.p1; ++pg, ++i) {
+          const int s = i % S::R;
+          if (i >= S::R &&
+              !wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
+            ok = false;
+            break;
+          }
+          const int phys = bt[pg];
+          const int row = (((un.l * p.P_phys + phys) * p.Hkv + un.kvh) * 2) * PS;
+          const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
+          mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
+          tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
+          tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
+        }
+      }
+      /* No copy may still be writing this CTA's shared memory when it exits. */
+      for (int k = (i > S::R ? i - S::R : 0); k < i; ++k)
+        wait_phase(smem_u32(&full[k % S::R]), (k / S::R) & 1, p, 2, false);
+    }
+    return;
+  }
+
+  /* ------------------------------------------------------- consumers ----- */
+  const int cw = warp - 1;
+  const int ct = threadIdx.x - 32;
+  const int NC = NCW * 32;
+  const int g = lane >> 2, t = lane & 3;
+  const int G = p.G;
+  const bool hv0 = (2 * t) < G, hv1 = (2 * t + 1) < G;
+  const uint64_t pol_keep = policy_evict_last();
+  const float NEG_INF = -INFINITY;
+
+  int i_base = 0, nunit = 0;
+  bool have_prev = false;
+  Unit prev{};
+  bool aborted = false;   // this warp gave up a wait
+  bool stopped = false;   // all consumer warps leave the unit loop together
+
+  auto finish = [&](const Unit &pv, int pv_slot) -> bool {
+    /* wait until every chunk of the item published its partial */
+    if (ct == 0) {
+      const int target = pv.C + p.extra_arrivals;
+      int okw = 1;
+      if (ld_acquire_gpu(&p.counters[pv.X]) < target) {
+        const long long t0 = globaltimer();
+        while (ld_acquire_gpu(&p.counters[pv.X]) < target) {
+          if (ld_volatile(&p.status[ST_ABORT])) { okw = 0; break; }
+          if (globaltimer() - t0 > p.spin_limit_ns) {
+            raise_status(p, MD_ERR_DEVICE_TIMEOUT, 3);
+            okw = 0;
+            break;
+          }
+          __nanosleep(100);
+        }
+      }
+      flag[2] = okw ? 0 : 1;
+    }
+    named_barrier(1, NC);
+    if (flag[2]) return false;
+    const float *base = p.partials + (size_t)pv.X * p.chunk_stride * PARTIAL_FLOATS;
+    if (ct < GP) {
+      float M = NEG_INF;
+      for (int j = 0; j < pv.C; ++j) M = fmaxf(M, __ldcg(base + (size_t)j * PARTIAL_FLOATS + ct));
+      const float Mr = (M == NEG_INF) ? 0.f : M;
+      float Z = 0.f;
+      for (int j = 0; j < pv.C; ++j) {
+        const float *pj = base + (size_t)j * PARTIAL_FLOATS;
+        Z += exp2f(__ldcg(pj + ct) - Mr) * __ldcg(pj + 8 + ct);
+      }
+      const float invZ = Z > 0.f ? 1.f / Z : 0.f;
+      fin[ct] = Mr;
+      fin[8 + ct] = invZ;
+      for (int j = 0; j < pv.C; ++j)
+        fac[j * GP + ct] = exp2f(__ldcg(base + (size_t)j * PARTIAL_FLOATS + ct) - Mr) * invZ;
+    }
+    named_barrier(1, NC);
+    /* this chunk's slice of the item's output O[h][d], h < G */
+    const int E = G * D;
+    const int lo = (int)(((long long)pv.j * E) / pv.C);
+    const int hi = (int)(((long long)(pv.j + 1) * E) / pv.C);
+    uint16_t *orow = p.out + (((size_t)pv.b * p.L + pv.l) * p.Hq + (size_t)pv.kvh * G) * D;
+    for (int e = lo + ct; e < hi; e += NC) {
+      const int h = e >> 7;
+      float acc = 0.f;
+      for (int j = 0; j < pv.C; ++j)
+        acc += fac[j * GP + h] * __ldcg(base + (size_t)j * PARTIAL_FLOATS + 16 + e);
+      __nv_bfloat16 v = __float2bfloat16_rn(acc);
+      orow[e] = *(uint16_t *)&v;
+    }
+    /* token masses of this chunk from its stored scores */
+    const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + pv_slot) * p.scratch_tokens * GP;
+    const int ntok = (pv.p1 - pv.p0) * PS;
+    const int nvalid = p.n_tokens[pv.b] - pv.p0 * PS;
+    const int32_t *bt = p.block_table + (size_t)pv.b * p.P_max;
+    float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
+    for (int tk = ct; tk < ntok; tk += NC) {
+      if (tk >= nvalid) continue;
+      const float4 s0 = *(const float4 *)(scr + (size_t)tk * GP);
+      const float4 s1 = *(const float4 *)(scr + (size_t)tk * GP + 4);
+      const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+      float m = 0.f;
+#pragma unroll
+      for (int h = 0; h < GP; ++h)
+        if (h < G) m += exp2f(sv[h] - fin[h]) * fin[8 + h];
+      const int pg = pv.p0 + tk / PS;
+      mrow[(size_t)bt[pg] * PS + (tk % PS)] = m;
+    }
+    named_barrier(1, NC);
+    if (ct == 0) {
+      const int old = atomicAdd(&p.counters[pv.X], 1);
+      if (old == 2 * pv.C - 1) atomicExch(&p.counters[pv.X], 0);
+    }
+    return true;
+  };
+
+  for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
+    const Unit un = decode_unit(p, u);
+    const int npg = un.p1 - un.p0;
+    const int slot = nunit & 1;
+    float *scr = p.scratch + ((size_t)blockIdx.x * 2 + slot) * p.scratch_tokens * GP;
+
+    /* Q^T fragments (B operand): head g, dims 16kk + {2t, 2t+1, 2t+8, 2t+9} */
+    uint32_t qf[8][2];
+    {
+      const uint16_t *qrow =
+          p.q + (((size_t)un.b * p.L + un.l) * p.Hq + (size_t)un.kvh * G + g) * D;
+      const bool gv = g < G;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        qf[kk][0] = gv ? *(const uint32_t *)(qrow + 16 * kk + 2 * t) : 0u;
+        qf[kk][1] = gv ? *(const uint32_t *)(qrow + 16 * kk + 8 + 2 * t) : 0u;
+      }
+    }
+    float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
+    float o[8][4];
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+    const int ntok_seq = p.n_tokens[un.b];
+    const int mi = lane >> 3, rr = lane & 7;
+
+    for (int jp = cw; jp < npg && !aborted; jp += NCW) {
+      const int gi = i_base + jp;
+      const int s = gi % S::R;
+      if (!wait_phase(smem_u32(&full[s]), (gi / S::R) & 1, p, 4, true)) {
+        aborted = true;
+        break;
+      }
+      const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
+      const int fill = ntok_seq - (un.p0 + jp) * PS;
+
+      float acc[S::NT][4];
+#pragma unroll
+      for (int tt = 0; tt < S::NT; ++tt) acc[tt][0] = acc[tt][1] = acc[tt][2] = acc[tt][3] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+#pragma unroll
+        for (int tt = 0; tt < S::NT; ++tt) {
+          uint32_t a0, a1, a2, a3;
+          ldmatrix_x4(swz<PS>(st, tt * 16 + (mi & 1) * 8 + rr, kk * 16 + (mi >> 1) * 8), a0, a1,
+                      a2, a3);
+          mma_bf16(acc[tt], a0, a1, a2, a3, qf[kk][0], qf[kk][1]);
+        }
+      }
+      /* scale to the exp2 domain, mask padded heads / unwritten tail slots,
+       * keep the raw scores for the mass pass */
+      float mx0 = NEG_INF, mx1 = NEG_INF;
+#pragma unroll
+      for (int tt = 0; tt < S::NT; ++tt) {
+        const int ta = tt * 16 + g, tb = ta + 8;
+        const bool va = ta < fill, vb = tb < fill;
+        acc[tt][0] = (va && hv0) ? acc[tt][0] * p.scale_log2 : NEG_INF;
+        acc[tt][1] = (va && hv1) ? acc[tt][1] * p.scale_log2 : NEG_INF;
+        acc[tt][2] = (vb && hv0) ? acc[tt][2] * p.scale_log2 : NEG_INF;
+        acc[tt][3] = (vb && hv1) ? acc[tt][3] * p.scale_log2 : NEG_INF;
+        st_v2_hint(scr + (size_t)(jp * PS + ta) * GP + 2 * t, acc[tt][0], acc[tt][1], pol_keep);
+        st_v2_hint(scr + (size_t)(jp * PS + tb) * GP + 2 * t, acc[tt][2], acc[tt][3], pol_keep);
+        mx0 = fmaxf(mx0, fmaxf(acc[tt][0], acc[tt][2]));
+        mx1 = fmaxf(mx1, fmaxf(acc[tt][1], acc[tt][3]));
+      }
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+      }
+      const float n0 = fmaxf(m0, mx0), n1 = fmaxf(m1, mx1);
+      const float r0 = (n0 == NEG_INF) ? 0.f : n0, r1 = (n1 == NEG_INF) ? 0.f : n1;
+      const float al0 = exp2f(m0 - r0), al1 = exp2f(m1 - r1);
+      m0 = n0;
+      m1 = n1;
+      l0 *= al0;
+      l1 *= al1;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        o[mt][0] *= al0;
+        o[mt][1] *= al1;
+        o[mt][2] *= al0;
+        o[mt][3] *= al1;
+      }
+#pragma unroll
+      for (int tt = 0; tt < S::NT; ++tt) {
+        const float p00 = exp2f(acc[tt][0] - r0), p01 = exp2f(acc[tt][1] - r1);
+        const float p10 = exp2f(acc[tt][2] - r0), p11 = exp2f(acc[tt][3] - r1);
+        l0 += p00 + p10;
+        l1 += p01 + p11;
+        const uint32_t b0 = movmatrix_trans(pack_bf16(p00, p01));
+        const uint32_t b1 = movmatrix_trans(pack_bf16(p10, p11));
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          uint32_t a0, a1, a2, a3;
+          ldmatrix_x4_trans(swz<PS>(st, PS + tt * 16 + (mi >> 1) * 8 + rr, mt * 16 + (mi & 1) * 8),
+                            a0, a1, a2, a3);
+          mma_bf16(o[mt], a0, a1, a2, a3, b0, b1);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
+    }
+
+    /* ---- merge the warps' partial softmax states, publish the unit's ---- */
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+    }
+    if (g == 0) {
+      wm[cw * 8 + 2 * t] = m0;
+      wm[cw * 8 + 2 * t + 1] = m1;
+      wl[cw * 8 + 2 * t] = l0;
+      wl[cw * 8 + 2 * t + 1] = l1;
+    }
+    {
+      float *wo = wO + (size_t)cw * GP * D;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        wo[(2 * t) * D + 16 * mt + g] = o[mt][0];
+        wo[(2 * t + 1) * D + 16 * mt + g] = o[mt][1];
+        wo[(2 * t) * D + 16 * mt + g + 8] = o[mt][2];
+        wo[(2 * t + 1) * D + 16 * mt + g + 8] = o[mt][3];
+      }
+    }
+    if (aborted) flag[0] = 1;
+    named_barrier(1, NC);
+    if (flag[0]) { stopped = true; break; }
+    float *part = p.partials + ((size_t)un.X * p.chunk_stride + un.j) * PARTIAL_FLOATS;
+    if (ct < GP) {
+      float M = NEG_INF;
+      for (int w = 0; w < NCW; ++w) M = fmaxf(M, wm[w * 8 + ct]);
+      const float Mr = (M == NEG_INF) ? 0.f : M;
+      float Lsum = 0.f;
+      for (int w = 0; w < NCW; ++w) Lsum += exp2f(wm[w * 8 + ct] - Mr) * wl[w * 8 + ct];
+      fin[ct] = Mr;
+      part[ct] = M;
+      part[8 + ct] = Lsum;
+    }
+    named_barrier(1, NC);
+    for (int e = ct; e < GP * D; e += NC) {
+      const int h = e >> 7;
+      float acc = 0.f;
+      for (int w = 0; w < NCW; ++w) acc += exp2f(wm[w * 8 + h] - fin[h]) * wO[(size_t)w * GP * D + e];
+      part[16 + e] = acc;
+    }
+    __threadfence();
+    named_barrier(1, NC);
+    if (ct == 0) {
+      atomicAdd(&p.counters[un.X], 1);
+      flag[1] = ld_volatile(&p.status[ST_ABORT]);
+    }
+    named_barrier(1, NC);
+    if (flag[1]) { stopped = true; break; }
+
+    if (have_prev && !finish(prev, (nunit - 1) & 1)) { stopped = true; break; }
+    prev = un;
+    have_prev = true;
+    i_base += npg;
+    ++nunit;
+  }
+  if (!stopped && have_prev) finish(prev, (nunit - 1) & 1);
+}
+
+template <int PS, int NCW>
+static cudaError_t prepare_impl() {
+  return cudaFuncSetAttribute(attn_mass_kernel<PS, NCW>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)AttnShape<PS, NCW>::SMEM);
+}
+
+template <int PS, int NCW>
+static int grid_limit_impl() {
+  int dev = 0, sms = 0, per_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (prepare_impl<PS, NCW>() != cudaSuccess) return 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_mass_kernel<PS, NCW>,
+                                                    AttnShape<PS, NCW>::THREADS,
+                                                    AttnShape<PS, NCW>::SMEM) != cudaSuccess)
+    return 0;
+  int g = sms * per_sm;
+  return g > MAX_GRID ? MAX_GRID : g;
+}
+
+template <int PS, int NCW>
+static cudaError_t launch_impl(const AttnParams &p, const CUtensorMap &tmap, int grid,
+                               cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(AttnShape<PS, NCW>::THREADS);
+  cfg.dynamicSmemBytes = AttnShape<PS, NCW>::SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attn_mass_kernel<PS, NCW>, p, tmap);
+}
+
+constexpr int NCW_DEFAULT = 4;
+
+cudaError_t attention_prepare(int ps) {
+  return ps == 16 ? prepare_impl<16, NCW_DEFAULT>() : prepare_impl<32, NCW_DEFAULT>();
+}
+
+int attention_grid_limit(int ps) {
+  return ps == 16 ? grid_limit_impl<16, NCW_DEFAULT>() : grid_limit_impl<32, NCW_DEFAULT>();
+}
+
+cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &tmap, int grid,
+                             cudaStream_t s) {
+  if (p.total_units == 0) return cudaSuccess;
+  return p.ps == 16 ? launch_impl<16, NCW_DEFAULT>(p, tmap, grid, s)
+                    : launch_impl<32, NCW_DEFAULT>(p, tmap, grid, s);
+}
+
+}  // namespace md

@@ -1,0 +1,911 @@
+/* Host side of libmemdecay: the C ABI of include/memdecay.h.
+ *
+ * The handle keeps an exact host mirror of the cache's bookkeeping (tokens
+ * and pages per sequence, pages holding a pinned token, the free-stack
+ * height, the decode step and the observation window).  Region labels are
+ * given on the host, so the number of evictable pages of every sequence is
+ * known here and the eviction counts, the free-stack offsets and the attention
+ * work split are computed without reading anything back from the GPU.  The
+ * kernels get these numbers by value in their launch parameters. */
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <vector>
+
+#include "md_internal.h"
+
+#define MD_API extern "C" __attribute__((visibility("default")))
+
+using namespace md;
+
+namespace {
+
+constexpr int N_STAGES = 5;
+constexpr int STAGE_APPEND = 0, STAGE_ATTN = 1, STAGE_FOLD = 2, STAGE_SCORE = 3,
+              STAGE_SELECT = 4;
+
+struct ProfRec {
+  int stage;
+  cudaEvent_t a, b;
+};
+
+struct HostMirror {
+  int64_t t = 0;
+  int window_steps = 0, window_batch = 0;
+  int mass_pending = 0, mass_batch = 0;
+  int64_t free_top = 0;
+};
+
+}  // namespace
+
+struct md_ctx {
+  md_config cfg;
+  Layout lay;
+  uint8_t *ws = nullptr;
+  cudaStream_t stream = nullptr;
+  CUtensorMap tmap;
+  int grid_limit = 0;
+  RegionTable reg;
+  HostMirror m;
+  std::vector<int64_t> n_tokens;
+  std::vector<int> n_pages, pinned_pages;
+  std::vector<uint8_t> tail_pinned;
+  bool poisoned = false;
+  std::string err;
+  long long spin_limit_ns = 2000000000LL;
+  int extra_arrivals = 0;
+  bool prof = false;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<ProfRec> pending;
+  double prof_ms[N_STAGES] = {0};
+  int64_t prof_n[N_STAGES] = {0};
+  std::vector<uint8_t> staging_host;
+};
+
+namespace {
+
+md_status fail(md_ctx *c, md_status s, const char *fmt, ...) __attribute__((format(printf, 3, 4)));
+md_status fail(md_ctx *c, md_status s, const char *fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    c->err = buf;
+  }
+  return s;
+}
+
+md_status cuda_fail(md_ctx *c, cudaError_t e, const char *what) {
+  if (c) {
+    c->err = std::string(what) + ": " + cudaGetErrorString(e);
+    c->poisoned = true;
+  }
+  return MD_ERR_CUDA;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+const char *check_config(const md_config &c) {
+  if (c.num_layers < 1 || c.num_layers > 255) return "num_layers must be in [1, 255]";
+  if (c.num_kv_heads < 1 || c.num_q_heads < c.num_kv_heads) return "bad head counts";
+  if (c.num_q_heads % c.num_kv_heads) return "num_q_heads must be a multiple of num_kv_heads";
+  if (c.num_q_heads / c.num_kv_heads > MD_MAX_GROUP) return "GQA group above 8 query heads";
+  if (c.head_dim != MD_HEAD_DIM) return "head_dim must be 128";
+  if (c.page_size != 16 && c.page_size != 32) return "page_size must be 16 or 32";
+  if (c.max_batch < 1 || c.max_batch > MD_MAX_BATCH) return "max_batch must be in [1, 256]";
+  if (c.max_pages_per_seq < 1 ||
+      (long long)c.max_pages_per_seq * c.page_size >
+          (long long)MD_MAX_CHUNKS * MD_MAX_CHUNK_TOKENS)
+    return "max_pages_per_seq out of range";
+  if (c.num_phys_pages < 1) return "num_phys_pages must be positive";
+  const long long rows =
+      (long long)c.num_layers * c.num_phys_pages * c.num_kv_heads * 2 * c.page_size;
+  if (rows >= (1LL << 31)) return "page pool too large (rows of K/V must stay below 2^31)";
+  if ((long long)c.num_phys_pages * c.page_size >= (1LL << 31)) return "too many token slots";
+  if (!(c.rho >= 0.f && c.rho <= 1.f) || !(c.gamma >= 0.f) || !isfinite(c.gamma))
+    return "rho must be in [0,1] and gamma >= 0";
+  if (!(c.tau_scale >= 0.f) || !isfinite(c.tau_scale)) return "tau_scale must be >= 0";
+  if (!(c.attn_weight >= 0.f) || !isfinite(c.attn_weight)) return "attn_weight must be >= 0";
+  if (c.score_mode != 0 && c.score_mode != 1) return "score_mode must be 0 or 1";
+  if (c.page_reduce != 0 && c.page_reduce != 1) return "page_reduce must be 0 or 1";
+  return nullptr;
+}
+
+void prof_begin(md_ctx *c, cudaEvent_t *a) {
+  *a = nullptr;
+  if (!c->prof) return;
+  if (c->ev_pool.empty()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return;
+    c->ev_pool.push_back(e);
+  }
+  *a = c->ev_pool.back();
+  c->ev_pool.pop_back();
+  cudaEventRecord(*a, c->stream);
+}
+
+void prof_end(md_ctx *c, int stage, cudaEvent_t a) {
+  if (!c->prof || !a) return;
+  cudaEvent_t b;
+  if (c->ev_pool.empty()) {
+    if (cudaEventCreate(&b) != cudaSuccess) {
+      c->ev_pool.push_back(a);
+      return;
+    }
+  } else {
+    b = c->ev_pool.back();
+    c->ev_pool.pop_back();
+  }
+  cudaEventRecord(b, c->stream);
+  c->pending.push_back({stage, a, b});
+}
+
+template <class T>
+T *ptr(md_ctx *c, size_t off) {
+  return (T *)(c->ws + off);
+}
+
+/* Pages of sequence b that can be evicted: everything but pinned pages and
+ * the page being written (the last one). */
+int evictable_pages(const md_ctx *c, int b) {
+  const int P = c->n_pages[b];
+  if (P == 0) return 0;
+  return P - c->pinned_pages[b] - (c->tail_pinned[b] ? 0 : 1);
+}
+
+/* Pinned-page bookkeeping for one appended token of region r. */
+void mirror_token(md_ctx *c, int b, int r) {
+  const int ps = c->cfg.page_size;
+  if (c->n_tokens[b] % ps == 0) {
+    c->n_pages[b] += 1;
+    c->tail_pinned[b] = 0;
+  }
+  if (c->reg.pinned[r] && !c->tail_pinned[b]) {
+    c->pinned_pages[b] += 1;
+    c->tail_pinned[b] = 1;
+  }
+  c->n_tokens[b] += 1;
+}
+
+int64_t cached_tokens(const md_ctx *c) {
+  int64_t s = 0;
+  for (auto v : c->n_tokens) s += v;
+  return s;
+}
+
+/* Window fold: add the pending per-(layer, head) mass rows into the window
+ * accumulator of every token that was attended in that step. */
+md_status launch_fold(md_ctx *c) {
+  ScoreParams sp;
+  memset(&sp, 0, sizeof(sp));
+  sp.mass = ptr<float>(c, c->lay.mass);
+  sp.window = ptr<float>(c, c->lay.window);
+  sp.region = ptr<uint8_t>(c, c->lay.region);
+  sp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  sp.slots = (long long)c->lay.slots;
+  sp.rows = c->cfg.num_layers * c->cfg.num_kv_heads;
+  sp.ps = c->cfg.page_size;
+  sp.P_max = c->cfg.max_pages_per_seq;
+  sp.fold_only = 1;
+  sp.n_seqs = c->m.mass_batch;
+  int tot = 0;
+  for (int b = 0; b < sp.n_seqs; ++b) {
+    sp.n_tokens[b] = (int)c->n_tokens[b];
+    sp.n_pages[b] = c->n_pages[b];
+    sp.page_start[b] = tot;
+    tot += c->n_pages[b];
+  }
+  sp.page_start[sp.n_seqs] = tot;
+  sp.total_pages = tot;
+  cudaEvent_t e0;
+  prof_begin(c, &e0);
+  cudaError_t err = launch_score(sp, c->stream);
+  prof_end(c, STAGE_FOLD, e0);
+  if (err != cudaSuccess) return cuda_fail(c, err, "fold launch");
+  c->m.mass_pending = 0;
+  return MD_OK;
+}
+
+/* Split every (sequence, layer, KV head) item's pages into chunks so that the
+ * persistent grid gets balanced rounds: minimise rounds x (largest chunk +
+ * a per-unit overhead), with at most MD_MAX_CHUNK_TOKENS tokens per chunk. */
+void plan_attention(const md_ctx *c, int batch, AttnParams &ap, int *grid) {
+  const int ps = c->cfg.page_size;
+  const int items = c->cfg.num_layers * c->cfg.num_kv_heads;
+  int Pmax = 1;
+  for (int b = 0; b < batch; ++b) Pmax = std::max(Pmax, c->n_pages[b]);
+  const int max_chunk_pages = std::max(1, c->lay.scratch_tokens / ps);
+  const int cmax = c->lay.chunk_stride;
+  double best = 1e300;
+  int bestT = 0;
+  for (int C = 1; C <= cmax; ++C) {
+    const int T = (Pmax + C - 1) / C;
+    if (T > max_chunk_pages) continue;
+    long long U = 0;
+    int maxpg = 0;
+    for (int b = 0; b < batch; ++b) {
+      const int P = c->n_pages[b];
+      if (P == 0) continue;
+      int ch = std::min(std::min((P + T - 1) / T, cmax), P);
+      U += (long long)items * ch;
+      maxpg = std::max(maxpg, (P + ch - 1) / ch);
+    }
+    const long long G = std::max(1LL, std::min<long long>(U, c->grid_limit));
+    const double rounds = (double)((U + G - 1) / G);
+    const double cost = rounds * (maxpg + 2.0);
+    if (cost < best - 1e-9) {
+      best = cost;
+      bestT = T;
+    }
+  }
+  long long U = 0;
+  for (int b = 0; b < batch; ++b) {
+    const int P = c->n_pages[b];
+    int ch = 0;
+    if (P > 0) ch = std::min(std::min((P + bestT - 1) / bestT, cmax), P);
+    ap.chunks[b] = ch;
+    ap.unit_start[b] = (int)U;
+    ap.n_pages[b] = P;
+    ap.n_tokens[b] = (int)c->n_tokens[b];
+    U += (long long)items * ch;
+  }
+  ap.unit_start[batch] = (int)U;
+  ap.total_units = (int)U;
+  ap.n_seqs = batch;
+  *grid = (int)std::max(1LL, std::min<long long>(U, c->grid_limit));
+}
+
+bool valid_region(int r) { return r >= 0 && r < MD_NUM_REGIONS; }
+
+}  // namespace
+
+/* ------------------------------------------------------------ layout ---- */
+size_t md::compute_layout(const md_config &c, Layout *lay) {
+  Layout L;
+  memset(&L, 0, sizeof(L));
+  const size_t ps = c.page_size;
+  L.slots = (size_t)c.num_phys_pages * ps;
+  L.n_items = (size_t)c.max_batch * c.num_layers * c.num_kv_heads;
+  L.scratch_tokens =
+      (int)std::min<long long>(MD_MAX_CHUNK_TOKENS, (long long)c.max_pages_per_seq * ps);
+  L.scratch_tokens = (L.scratch_tokens + 15) / 16 * 16;
+  L.chunk_stride = std::min(MD_MAX_CHUNKS, c.max_pages_per_seq);
+  size_t off = 0;
+  auto take = [&](size_t bytes, size_t align) {
+    off = align_up(off, align);
+    size_t o = off;
+    off += bytes;
+    return o;
+  };
+  L.status = take(ST_WORDS * 4 * 4, 256);
+  L.pool = take((size_t)c.num_layers * c.num_phys_pages * c.num_kv_heads * 2 * ps * D * 2, 1024);
+  L.block_table = take((size_t)c.max_batch * c.max_pages_per_seq * 4, 256);
+  L.page_score = take((size_t)c.max_batch * c.max_pages_per_seq * 4, 256);
+  L.free_stack = take((size_t)c.num_phys_pages * 4, 256);
+  L.region = take(L.slots, 256);
+  L.a = take(L.slots * 4, 256);
+  L.t_ref = take(L.slots * 4, 256);
+  L.window = take(L.slots * 4, 256);
+  L.ahat = take(L.slots * 4, 256);
+  L.prio = take(L.slots * 4, 256);
+  L.mass = take((size_t)c.num_layers * c.num_kv_heads * L.slots * 4, 256);
+  L.scratch = take((size_t)MAX_GRID * 2 * L.scratch_tokens * GP * 4, 256);
+  L.partials = take(L.n_items * L.chunk_stride * PARTIAL_FLOATS * 4, 256);
+  L.counters = take(L.n_items * 4, 256);
+  L.evict_list = take((size_t)c.max_batch * c.max_pages_per_seq * 4, 256);
+  L.staging_regions = take((size_t)c.max_pages_per_seq * ps, 256);
+  L.staging_steps = take((size_t)c.max_pages_per_seq * ps * 4, 256);
+  L.total = align_up(off, 256);
+  if (lay) *lay = L;
+  return L.total;
+}
+
+/* ------------------------------------------------------------- C ABI ---- */
+MD_API size_t md_workspace_size(const md_config *cfg) {
+  if (!cfg || check_config(*cfg)) return 0;
+  return compute_layout(*cfg, nullptr);
+}
+
+MD_API md_status md_create(const md_config *cfg, md_ctx **out) {
+  if (!cfg || !out) return MD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (check_config(*cfg)) return MD_ERR_INVALID_ARG;
+  Layout lay;
+  const size_t need = compute_layout(*cfg, &lay);
+  if (!cfg->workspace || ((uintptr_t)cfg->workspace & 1023) || cfg->workspace_bytes < need)
+    return MD_ERR_WORKSPACE;
+  md_ctx *c = new md_ctx();
+  c->cfg = *cfg;
+  c->lay = lay;
+  c->ws = (uint8_t *)cfg->workspace;
+  c->stream = (cudaStream_t)cfg->stream;
+  const int B = cfg->max_batch;
+  c->n_tokens.assign(B, 0);
+  c->n_pages.assign(B, 0);
+  c->pinned_pages.assign(B, 0);
+  c->tail_pinned.assign(B, 0);
+  for (int r = 0; r < 8; ++r) {
+    c->reg.base[r] = 0.f;
+    c->reg.half_life[r] = INFINITY;
+    c->reg.pinned[r] = 0;
+  }
+  c->m.free_top = cfg->num_phys_pages;
+
+  cudaError_t e = attention_prepare(cfg->page_size);
+  if (e != cudaSuccess) {
+    delete c;
+    return MD_ERR_CUDA;
+  }
+  c->grid_limit = attention_grid_limit(cfg->page_size);
+  if (c->grid_limit <= 0) {
+    delete c;
+    return MD_ERR_CUDA;
+  }
+  /* TMA descriptor over the pool viewed as [rows][128] bf16, rows = (layer,
+   * page, KV head, K|V, token); one box = one page's K and V rows x 64 dims,
+   * 128-byte swizzled. */
+  void *fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+  if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) {
+    delete c;
+    return MD_ERR_CUDA;
+  }
+  typedef CUresult (*EncodeFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                               const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                               const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                               CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  const cuuint64_t rows = (cuuint64_t)cfg->num_layers * cfg->num_phys_pages *
+                          cfg->num_kv_heads * 2 * cfg->page_size;
+  cuuint64_t dims[2] = {(cuuint64_t)D, rows};
+  cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)(2 * cfg->page_size)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult cr = ((EncodeFn)fn)(&c->tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->ws + lay.pool,
+                               dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS) {
+    delete c;
+    return MD_ERR_CUDA;
+  }
+  e = cudaMemsetAsync(c->ws, 0, need, c->stream);
+  if (e == cudaSuccess)
+    e = launch_init(ptr<int32_t>(c, lay.free_stack), cfg->num_phys_pages, ptr<int>(c, lay.status),
+                    ptr<int>(c, lay.counters), lay.n_items, c->stream);
+  if (e != cudaSuccess) {
+    delete c;
+    return MD_ERR_CUDA;
+  }
+  *out = c;
+  return MD_OK;
+}
+
+MD_API md_status md_set_region_params(md_ctx *c, int region, float base, float half_life,
+                                      int pinned) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (!valid_region(region)) return fail(c, MD_ERR_INVALID_ARG, "region %d out of range", region);
+  if (!(base >= 0.f) || !isfinite(base))
+    return fail(c, MD_ERR_INVALID_ARG, "base priority must be finite and >= 0");
+  if (!(half_life > 0.f)) return fail(c, MD_ERR_INVALID_ARG, "half-life must be > 0 (or +inf)");
+  const int pin = pinned ? 1 : 0;
+  if (pin != c->reg.pinned[region] && cached_tokens(c) > 0)
+    return fail(c, MD_ERR_STATE, "pinned flag can only change while the cache is empty");
+  c->reg.base[region] = base;
+  c->reg.half_life[region] = half_life;
+  c->reg.pinned[region] = pin;
+  return MD_OK;
+}
+
+MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regions_host,
+                                  const int32_t *steps_host, const void *k_dev,
+                                  const void *v_dev) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  const md_config &cf = c->cfg;
+  if (seq < 0 || seq >= cf.max_batch) return fail(c, MD_ERR_INVALID_ARG, "seq out of range");
+  if (n < 0) return fail(c, MD_ERR_INVALID_ARG, "negative token count");
+  if (n == 0) return MD_OK;
+  if (!regions_host || !k_dev || !v_dev) return fail(c, MD_ERR_INVALID_ARG, "null pointer");
+  for (int i = 0; i < n; ++i)
+    if (!valid_region(regions_host[i])) return fail(c, MD_ERR_INVALID_ARG, "bad region label");
+  if (steps_host)
+    for (int i = 0; i < n; ++i)
+      if (steps_host[i] > c->m.t) return fail(c, MD_ERR_INVALID_ARG, "insertion step in the future");
+  const int ps = cf.page_size;
+  const long long tok_after = c->n_tokens[seq] + (long long)n;
+  const long long pages_after = (tok_after + ps - 1) / ps;
+  const long long new_pages = pages_after - c->n_pages[seq];
+  if (pages_after > cf.max_pages_per_seq)
+    return fail(c, MD_ERR_CAPACITY, "sequence %d would need %lld pages (max %d)", seq,
+                pages_after, cf.max_pages_per_seq);
+  if (new_pages > c->m.free_top)
+    return fail(c, MD_ERR_CAPACITY, "page pool exhausted (%lld free, %lld needed)",
+                (long long)c->m.free_top, new_pages);
+  if (c->m.mass_pending) {
+    md_status st = launch_fold(c);
+    if (st != MD_OK) return st;
+  }
+  cudaError_t e = cudaMemcpyAsync(c->ws + c->lay.staging_regions, regions_host, (size_t)n,
+                                  cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess && steps_host)
+    e = cudaMemcpyAsync(c->ws + c->lay.staging_steps, steps_host, (size_t)n * 4,
+                        cudaMemcpyHostToDevice, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "staging copy");
+  AppendParams ap;
+  memset(&ap, 0, sizeof(ap));
+  ap.pool = ptr<uint16_t>(c, c->lay.pool);
+  ap.block_table = ptr<int32_t>(c, c->lay.block_table);
+  ap.free_stack = ptr<int32_t>(c, c->lay.free_stack);
+  ap.region = ptr<uint8_t>(c, c->lay.region);
+  ap.a = ptr<float>(c, c->lay.a);
+  ap.window = ptr<float>(c, c->lay.window);
+  ap.ahat = ptr<float>(c, c->lay.ahat);
+  ap.prio = ptr<float>(c, c->lay.prio);
+  ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
+  ap.k_src = (const uint16_t *)k_dev;
+  ap.v_src = (const uint16_t *)v_dev;
+  ap.sb = 0;
+  ap.sl = (long long)cf.num_kv_heads * n * D;
+  ap.sh = (long long)n * D;
+  ap.si = D;
+  ap.regions_dev = ptr<uint8_t>(c, c->lay.staging_regions);
+  ap.steps_dev = steps_host ? ptr<int32_t>(c, c->lay.staging_steps) : nullptr;
+  ap.L = cf.num_layers;
+  ap.Hkv = cf.num_kv_heads;
+  ap.ps = ps;
+  ap.P_phys = cf.num_phys_pages;
+  ap.P_max = cf.max_pages_per_seq;
+  ap.n_seqs = 1;
+  ap.n_per_seq = n;
+  ap.seq0 = seq;
+  ap.insert_step = (int)c->m.t;
+  ap.tok0[0] = (int)c->n_tokens[seq];
+  ap.pop_base[0] = (int)(c->m.free_top - 1);
+  cudaEvent_t e0;
+  prof_begin(c, &e0);
+  e = launch_append(ap, c->stream);
+  prof_end(c, STAGE_APPEND, e0);
+  if (e != cudaSuccess) return cuda_fail(c, e, "append launch");
+  for (int i = 0; i < n; ++i) mirror_token(c, seq, regions_host[i]);
+  c->m.free_top -= new_pages;
+  return MD_OK;
+}
+
+MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const void *k_new,
+                                const void *v_new, const uint8_t *new_region_host,
+                                void *out_dev) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  const md_config &cf = c->cfg;
+  if (batch < 1 || batch > cf.max_batch) return fail(c, MD_ERR_INVALID_ARG, "batch out of range");
+  if (!q_dev || !k_new || !v_new || !new_region_host || !out_dev)
+    return fail(c, MD_ERR_INVALID_ARG, "null pointer");
+  if (c->m.window_steps > 0 && batch != c->m.window_batch)
+    return fail(c, MD_ERR_INVALID_ARG, "batch changed inside an observation window");
+  const int ps = cf.page_size;
+  long long need_total = 0;
+  for (int b = 0; b < batch; ++b) {
+    if (!valid_region(new_region_host[b])) return fail(c, MD_ERR_INVALID_ARG, "bad region label");
+    const int need = (c->n_tokens[b] % ps == 0) ? 1 : 0;
+    if (c->n_pages[b] + need > cf.max_pages_per_seq)
+      return fail(c, MD_ERR_CAPACITY, "sequence %d block table full", b);
+    need_total += need;
+  }
+  if (need_total > c->m.free_top) return fail(c, MD_ERR_CAPACITY, "page pool exhausted");
+  if (c->m.t + 1 >= (1LL << 31)) return fail(c, MD_ERR_STATE, "step counter overflow");
+
+  if (c->m.mass_pending) {
+    md_status st = launch_fold(c);
+    if (st != MD_OK) return st;
+  }
+  c->m.t += 1;
+  /* stage 0: append the new tokens */
+  AppendParams ap;
+  memset(&ap, 0, sizeof(ap));
+  ap.pool = ptr<uint16_t>(c, c->lay.pool);
+  ap.block_table = ptr<int32_t>(c, c->lay.block_table);
+  ap.free_stack = ptr<int32_t>(c, c->lay.free_stack);
+  ap.region = ptr<uint8_t>(c, c->lay.region);
+  ap.a = ptr<float>(c, c->lay.a);
+  ap.window = ptr<float>(c, c->lay.window);
+  ap.ahat = ptr<float>(c, c->lay.ahat);
+  ap.prio = ptr<float>(c, c->lay.prio);
+  ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
+  ap.k_src = (const uint16_t *)k_new;
+  ap.v_src = (const uint16_t *)v_new;
+  ap.sb = (long long)cf.num_layers * cf.num_kv_heads * D;
+  ap.sl = (long long)cf.num_kv_heads * D;
+  ap.sh = D;
+  ap.si = 0;
+  ap.L = cf.num_layers;
+  ap.Hkv = cf.num_kv_heads;
+  ap.ps = ps;
+  ap.P_phys = cf.num_phys_pages;
+  ap.P_max = cf.max_pages_per_seq;
+  ap.n_seqs = batch;
+  ap.n_per_seq = 1;
+  ap.seq0 = 0;
+  ap.insert_step = (int)c->m.t;
+  long long popped = 0;
+  for (int b = 0; b < batch; ++b) {
+    ap.tok0[b] = (int)c->n_tokens[b];
+    ap.pop_base[b] = (int)(c->m.free_top - 1 - popped);
+    ap.regions_param[b] = new_region_host[b];
+    if (c->n_tokens[b] % ps == 0) popped += 1;
+  }
+  cudaEvent_t e0;
+  prof_begin(c, &e0);
+  cudaError_t e = launch_append(ap, c->stream);
+  prof_end(c, STAGE_APPEND, e0);
+  if (e != cudaSuccess) return cuda_fail(c, e, "append launch");
+  for (int b = 0; b < batch; ++b) mirror_token(c, b, new_region_host[b]);
+  c->m.free_top -= popped;
+
+  /* stage 1: attention + mass */
+  AttnParams atp;
+  memset(&atp, 0, sizeof(atp));
+  atp.q = (const uint16_t *)q_dev;
+  atp.out = (uint16_t *)out_dev;
+  atp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  atp.mass = ptr<float>(c, c->lay.mass);
+  atp.scratch = ptr<float>(c, c->lay.scratch);
+  atp.partials = ptr<float>(c, c->lay.partials);
+  atp.counters = ptr<int>(c, c->lay.counters);
+  atp.status = ptr<int>(c, c->lay.status);
+  atp.L = cf.num_layers;
+  atp.Hq = cf.num_q_heads;
+  atp.Hkv = cf.num_kv_heads;
+  atp.G = cf.num_q_heads / cf.num_kv_heads;
+  atp.ps = ps;
+  atp.P_phys = cf.num_phys_pages;
+  atp.P_max = cf.max_pages_per_seq;
+  atp.slots = (long long)c->lay.slots;
+  atp.scratch_tokens = c->lay.scratch_tokens;
+  atp.chunk_stride = c->lay.chunk_stride;
+  atp.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
+  atp.spin_limit_ns = c->spin_limit_ns;
+  atp.extra_arrivals = c->extra_arrivals;
+  c->extra_arrivals = 0;
+  int grid = 1;
+  plan_attention(c, batch, atp, &grid);
+  prof_begin(c, &e0);
+  e = launch_attention(atp, c->tmap, grid, c->stream);
+  prof_end(c, STAGE_ATTN, e0);
+  if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
+  c->m.mass_pending = 1;
+  c->m.mass_batch = batch;
+  c->m.window_steps += 1;
+  c->m.window_batch = batch;
+  return MD_OK;
+}
+
+MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *n_evicted_host,
+                          int32_t *evicted_ids_dev) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  const md_config &cf = c->cfg;
+  if (batch < 1 || batch > cf.max_batch) return fail(c, MD_ERR_INVALID_ARG, "batch out of range");
+  if (!budget) return fail(c, MD_ERR_INVALID_ARG, "null budget");
+  if (c->m.window_steps > 0 && batch != c->m.window_batch)
+    return fail(c, MD_ERR_INVALID_ARG, "batch differs from the observation window's");
+  for (int b = 0; b < batch; ++b)
+    if (budget[b] < 0) return fail(c, MD_ERR_INVALID_ARG, "negative budget");
+  const int ps = cf.page_size;
+
+  /* stages 2-3 */
+  ScoreParams sp;
+  memset(&sp, 0, sizeof(sp));
+  sp.mass = ptr<float>(c, c->lay.mass);
+  sp.window = ptr<float>(c, c->lay.window);
+  sp.a = ptr<float>(c, c->lay.a);
+  sp.ahat = ptr<float>(c, c->lay.ahat);
+  sp.prio = ptr<float>(c, c->lay.prio);
+  sp.page_score = ptr<float>(c, c->lay.page_score);
+  sp.t_ref = ptr<int32_t>(c, c->lay.t_ref);
+  sp.region = ptr<uint8_t>(c, c->lay.region);
+  sp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  sp.slots = (long long)c->lay.slots;
+  sp.rows = cf.num_layers * cf.num_kv_heads;
+  sp.ps = ps;
+  sp.P_max = cf.max_pages_per_seq;
+  sp.fold_only = 0;
+  sp.observe = c->m.window_steps > 0 ? 1 : 0;
+  sp.mass_pending = c->m.mass_pending;
+  sp.norm = (float)((double)std::max(1, c->m.window_steps) * cf.num_layers * cf.num_q_heads);
+  sp.t = (int)c->m.t;
+  sp.rho = cf.rho;
+  sp.gamma = cf.gamma;
+  sp.tau_scale = cf.tau_scale;
+  sp.alpha = cf.attn_weight;
+  sp.score_mode = cf.score_mode;
+  sp.page_reduce = cf.page_reduce;
+  sp.keep_prio = 1;
+  sp.reg = c->reg;
+  sp.n_seqs = batch;
+  int tot = 0;
+  for (int b = 0; b < batch; ++b) {
+    sp.n_tokens[b] = (int)c->n_tokens[b];
+    sp.n_pages[b] = c->n_pages[b];
+    sp.page_start[b] = tot;
+    tot += c->n_pages[b];
+  }
+  sp.page_start[batch] = tot;
+  sp.total_pages = tot;
+  cudaEvent_t e0;
+  prof_begin(c, &e0);
+  cudaError_t e = launch_score(sp, c->stream);
+  prof_end(c, STAGE_SCORE, e0);
+  if (e != cudaSuccess) return cuda_fail(c, e, "score launch");
+
+  /* stage 4 */
+  SelectParams sel;
+  memset(&sel, 0, sizeof(sel));
+  sel.page_score = ptr<float>(c, c->lay.page_score);
+  sel.block_table = ptr<int32_t>(c, c->lay.block_table);
+  sel.free_stack = ptr<int32_t>(c, c->lay.free_stack);
+  sel.evict_list = ptr<int32_t>(c, c->lay.evict_list);
+  sel.user_evicted = evicted_ids_dev;
+  sel.status = ptr<int>(c, c->lay.status);
+  sel.P_max = cf.max_pages_per_seq;
+  sel.n_seqs = batch;
+  sel.top = (int)c->m.free_top;
+  bool warn = false;
+  int any = 0, pushed = 0;
+  std::vector<int> ev(batch);
+  for (int b = 0; b < batch; ++b) {
+    const int P = c->n_pages[b];
+    const int want = std::max(0, P - budget[b]);
+    const int can = std::max(0, evictable_pages(c, b));
+    ev[b] = std::min(want, can);
+    if (ev[b] < want) warn = true;
+    sel.n_pages[b] = P;
+    sel.n_evict[b] = ev[b];
+    sel.push_off[b] = pushed;
+    pushed += ev[b];
+    any |= ev[b] > 0;
+  }
+  if (any || evicted_ids_dev) {
+    prof_begin(c, &e0);
+    e = launch_select(sel, c->stream);
+    prof_end(c, STAGE_SELECT, e0);
+    if (e != cudaSuccess) return cuda_fail(c, e, "select launch");
+  }
+  for (int b = 0; b < batch; ++b) {
+    c->n_pages[b] -= ev[b];
+    c->n_tokens[b] -= (int64_t)ev[b] * ps;
+    if (n_evicted_host) n_evicted_host[b] = ev[b];
+  }
+  c->m.free_top += pushed;
+  c->m.window_steps = 0;
+  c->m.mass_pending = 0;
+  return warn ? MD_WARN_OVER_BUDGET : MD_OK;
+}
+
+MD_API md_status md_sync(md_ctx *c) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "stream synchronize");
+  int st[ST_WORDS];
+  e = cudaMemcpy(st, c->ws + c->lay.status, sizeof(st), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(c, e, "status read");
+  if (st[ST_CODE] != 0) {
+    c->poisoned = true;
+    char buf[160];
+    snprintf(buf, sizeof(buf), "device status %d (site %d)", st[ST_CODE], st[ST_DIAG]);
+    c->err = buf;
+    return (md_status)st[ST_CODE];
+  }
+  return MD_OK;
+}
+
+MD_API md_status md_destroy(md_ctx *c) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  cudaStreamSynchronize(c->stream);
+  for (auto &r : c->pending) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : c->ev_pool) cudaEventDestroy(e);
+  delete c;
+  return MD_OK;
+}
+
+namespace {
+bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
+  const md_config &cf = c->cfg;
+  const Layout &L = c->lay;
+  const size_t bt = (size_t)cf.max_batch * cf.max_pages_per_seq * 4;
+  switch (what) {
+    case MD_STATE_BLOCK_TABLE: *off = L.block_table; *bytes = bt; return true;
+    case MD_STATE_PAGE_SCORE: *off = L.page_score; *bytes = bt; return true;
+    case MD_STATE_TOKEN_PRIO: *off = L.prio; *bytes = L.slots * 4; return true;
+    case MD_STATE_A: *off = L.a; *bytes = L.slots * 4; return true;
+    case MD_STATE_T_REF: *off = L.t_ref; *bytes = L.slots * 4; return true;
+    case MD_STATE_AHAT: *off = L.ahat; *bytes = L.slots * 4; return true;
+    case MD_STATE_FREE: *off = L.free_stack; *bytes = (size_t)cf.num_phys_pages * 4; return true;
+    case MD_STATE_REGION: *off = L.region; *bytes = L.slots; return true;
+    case MD_STATE_WINDOW: *off = L.window; *bytes = L.slots * 4; return true;
+    case MD_STATE_MASS:
+      *off = L.mass;
+      *bytes = (size_t)cf.num_layers * cf.num_kv_heads * L.slots * 4;
+      return true;
+    case MD_STATE_POOL:
+      *off = L.pool;
+      *bytes = (size_t)cf.num_layers * cf.num_phys_pages * cf.num_kv_heads * 2 * cf.page_size * D * 2;
+      return true;
+  }
+  return false;
+}
+const int SAVED[] = {MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A,
+                     MD_STATE_T_REF,       MD_STATE_AHAT,       MD_STATE_FREE,       MD_STATE_REGION,
+                     MD_STATE_WINDOW};
+}  // namespace
+
+MD_API md_status md_get_state(md_ctx *c, int what, void *dst, size_t bytes) {
+  if (!c || !dst) return MD_ERR_INVALID_ARG;
+  size_t off, n;
+  if (!state_array(c, what, &off, &n)) return fail(c, MD_ERR_INVALID_ARG, "unknown state array");
+  if (bytes != n) return fail(c, MD_ERR_INVALID_ARG, "state array is %zu bytes, not %zu", n, bytes);
+  cudaError_t e = cudaMemcpyAsync(dst, c->ws + off, n, cudaMemcpyDeviceToDevice, c->stream);
+  return e == cudaSuccess ? MD_OK : cuda_fail(c, e, "state copy");
+}
+
+MD_API md_status md_set_state(md_ctx *c, int what, const void *src, size_t bytes) {
+  if (!c || !src) return MD_ERR_INVALID_ARG;
+  if (what != MD_STATE_BLOCK_TABLE && what != MD_STATE_FREE && what != MD_STATE_A &&
+      what != MD_STATE_T_REF)
+    return fail(c, MD_ERR_INVALID_ARG, "state array is read-only");
+  size_t off, n;
+  state_array(c, what, &off, &n);
+  if (bytes != n) return fail(c, MD_ERR_INVALID_ARG, "state array is %zu bytes, not %zu", n, bytes);
+  cudaError_t e = cudaMemcpyAsync(c->ws + off, src, n, cudaMemcpyDeviceToDevice, c->stream);
+  return e == cudaSuccess ? MD_OK : cuda_fail(c, e, "state copy");
+}
+
+MD_API md_status md_query(const md_ctx *c, int what, int seq, int64_t *out) {
+  if (!c || !out) return MD_ERR_INVALID_ARG;
+  const bool per_seq = what == MD_QUERY_TOKENS || what == MD_QUERY_PAGES || what == MD_QUERY_PINNED_PAGES;
+  if (per_seq && (seq < 0 || seq >= c->cfg.max_batch)) return MD_ERR_INVALID_ARG;
+  switch (what) {
+    case MD_QUERY_TOKENS: *out = c->n_tokens[seq]; return MD_OK;
+    case MD_QUERY_PAGES: *out = c->n_pages[seq]; return MD_OK;
+    case MD_QUERY_FREE_TOP: *out = c->m.free_top; return MD_OK;
+    case MD_QUERY_STEP: *out = c->m.t; return MD_OK;
+    case MD_QUERY_WINDOW: *out = c->m.window_steps; return MD_OK;
+    case MD_QUERY_PINNED_PAGES: *out = c->pinned_pages[seq]; return MD_OK;
+  }
+  return MD_ERR_INVALID_ARG;
+}
+
+namespace {
+size_t host_blob_bytes(const md_ctx *c) {
+  const size_t B = c->cfg.max_batch;
+  return sizeof(HostMirror) + sizeof(RegionTable) + B * (8 + 4 + 4 + 1);
+}
+}  // namespace
+
+MD_API md_status md_state_bytes(const md_ctx *c, size_t *dev_bytes, size_t *host_bytes) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  size_t tot = 0, off, n;
+  for (int w : SAVED) {
+    state_array(c, w, &off, &n);
+    tot += n;
+  }
+  if (dev_bytes) *dev_bytes = tot;
+  if (host_bytes) *host_bytes = host_blob_bytes(c);
+  return MD_OK;
+}
+
+MD_API md_status md_save_state(md_ctx *c, void *dst_dev, void *host_blob) {
+  if (!c || !dst_dev || !host_blob) return MD_ERR_INVALID_ARG;
+  if (c->m.window_steps != 0 || c->m.mass_pending)
+    return fail(c, MD_ERR_STATE, "checkpoint only between observation windows");
+  size_t pos = 0, off, n;
+  for (int w : SAVED) {
+    state_array(c, w, &off, &n);
+    cudaError_t e = cudaMemcpyAsync((uint8_t *)dst_dev + pos, c->ws + off, n,
+                                    cudaMemcpyDeviceToDevice, c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "checkpoint copy");
+    pos += n;
+  }
+  uint8_t *h = (uint8_t *)host_blob;
+  const size_t B = c->cfg.max_batch;
+  memcpy(h, &c->m, sizeof(HostMirror));
+  h += sizeof(HostMirror);
+  memcpy(h, &c->reg, sizeof(RegionTable));
+  h += sizeof(RegionTable);
+  memcpy(h, c->n_tokens.data(), B * 8);
+  h += B * 8;
+  memcpy(h, c->n_pages.data(), B * 4);
+  h += B * 4;
+  memcpy(h, c->pinned_pages.data(), B * 4);
+  h += B * 4;
+  memcpy(h, c->tail_pinned.data(), B);
+  return MD_OK;
+}
+
+MD_API md_status md_load_state(md_ctx *c, const void *src_dev, const void *host_blob) {
+  if (!c || !src_dev || !host_blob) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  size_t pos = 0, off, n;
+  for (int w : SAVED) {
+    state_array(c, w, &off, &n);
+    cudaError_t e = cudaMemcpyAsync(c->ws + off, (const uint8_t *)src_dev + pos, n,
+                                    cudaMemcpyDeviceToDevice, c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "restore copy");
+    pos += n;
+  }
+  const uint8_t *h = (const uint8_t *)host_blob;
+  const size_t B = c->cfg.max_batch;
+  memcpy(&c->m, h, sizeof(HostMirror));
+  h += sizeof(HostMirror);
+  memcpy(&c->reg, h, sizeof(RegionTable));
+  h += sizeof(RegionTable);
+  memcpy(c->n_tokens.data(), h, B * 8);
+  h += B * 8;
+  memcpy(c->n_pages.data(), h, B * 4);
+  h += B * 4;
+  memcpy(c->pinned_pages.data(), h, B * 4);
+  h += B * 4;
+  memcpy(c->tail_pinned.data(), h, B);
+  return MD_OK;
+}
+
+MD_API md_status md_profile_enable(md_ctx *c, int enable) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  c->prof = enable != 0;
+  if (c->prof) {
+    for (int s = 0; s < N_STAGES; ++s) {
+      c->prof_ms[s] = 0;
+      c->prof_n[s] = 0;
+    }
+  }
+  return MD_OK;
+}
+
+MD_API md_status md_profile_read(md_ctx *c, double *ms, int64_t *launches, int n_stages) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "stream synchronize");
+  for (auto &r : c->pending) {
+    float x = 0.f;
+    if (cudaEventElapsedTime(&x, r.a, r.b) == cudaSuccess) {
+      c->prof_ms[r.stage] += x;
+      c->prof_n[r.stage] += 1;
+    }
+    c->ev_pool.push_back(r.a);
+    c->ev_pool.push_back(r.b);
+  }
+  c->pending.clear();
+  for (int s = 0; s < n_stages && s < N_STAGES; ++s) {
+    if (ms) ms[s] = c->prof_ms[s];
+    if (launches) launches[s] = c->prof_n[s];
+  }
+  return MD_OK;
+}
+
+MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (key == MD_DEBUG_SPIN_LIMIT_NS) {
+    if (value < 1000) return fail(c, MD_ERR_INVALID_ARG, "spin limit below 1 us");
+    c->spin_limit_ns = (long long)value;
+    return MD_OK;
+  }
+  if (key == MD_DEBUG_EXTRA_ARRIVALS) {
+    if (value < 0 || value > 1000) return fail(c, MD_ERR_INVALID_ARG, "extra arrivals out of range");
+    c->extra_arrivals = (int)value;
+    return MD_OK;
+  }
+  return fail(c, MD_ERR_INVALID_ARG, "unknown debug key");
+}
+
+MD_API const char *md_last_error(const md_ctx *c) { return c ? c->err.c_str() : "null handle"; }

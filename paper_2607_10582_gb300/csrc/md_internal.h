@@ -1,0 +1,130 @@
+/* Internal declarations of libmemdecay: workspace layout, launch parameters
+ * (passed by value; per-sequence counts come from the exact host mirror) and
+ * the launchers of the four kernels. */
+#ifndef MD_INTERNAL_H
+#define MD_INTERNAL_H
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/memdecay.h"
+
+namespace md {
+
+constexpr int D = MD_HEAD_DIM;
+constexpr int GP = MD_MAX_GROUP;            // query heads per KV head, padded
+constexpr int PARTIAL_FLOATS = 1088;        // m[8] l[8] O[8][128], padded to 256 B
+constexpr int MAX_GRID = 256;               // persistent attention CTAs (>= SM count)
+
+enum DevStatus { ST_CODE = 0, ST_ABORT = 1, ST_DIAG = 2, ST_WORDS = 8 };
+
+struct RegionTable {
+  float base[8];
+  float half_life[8];
+  int pinned[8];
+};
+
+/* Byte offsets of every array inside the caller's workspace. */
+struct Layout {
+  size_t pool, block_table, page_score, free_stack, region, a, t_ref, window, ahat, prio, mass,
+      scratch, partials, counters, evict_list, staging_regions, staging_steps, status, total;
+  size_t slots, n_items;
+  int scratch_tokens, chunk_stride;
+};
+
+size_t compute_layout(const md_config &c, Layout *lay);
+
+/* ------------------------------------------------------------- append --- */
+struct AppendParams {
+  uint16_t *pool;
+  int32_t *block_table;
+  const int32_t *free_stack;
+  uint8_t *region;
+  float *a, *window, *ahat, *prio;
+  int32_t *t_ref;
+  const uint16_t *k_src, *v_src;
+  long long sb, sl, sh, si;              // element strides of the source (seq, layer, head, token)
+  const uint8_t *regions_dev;            // per token (prefill) or null
+  const int32_t *steps_dev;              // per token (prefill) or null
+  int L, Hkv, ps, P_phys, P_max;
+  int n_seqs, n_per_seq, seq0, insert_step;
+  int tok0[MD_MAX_BATCH];                // cached tokens before this append
+  int pop_base[MD_MAX_BATCH];            // free-stack index of the first page taken
+  uint8_t regions_param[MD_MAX_BATCH];   // decode: region of each new token
+};
+cudaError_t launch_append(const AppendParams &p, cudaStream_t s);
+
+/* ---------------------------------------------------------- attention --- */
+struct AttnParams {
+  const uint16_t *q;
+  uint16_t *out;
+  const int32_t *block_table;
+  float *mass;         // [L*Hkv][slots]
+  float *scratch;      // [grid][2][scratch_tokens][8]
+  float *partials;     // [items][chunk_stride][PARTIAL_FLOATS]
+  int *counters;       // [items]
+  int *status;         // sticky device status words
+  int L, Hq, Hkv, G, ps, P_phys, P_max;
+  long long slots;
+  int scratch_tokens;  // scratch row capacity per CTA slot (tokens)
+  int chunk_stride;    // partial slots reserved per item
+  float scale_log2;    // log2(e) / sqrt(D)
+  long long spin_limit_ns;
+  int extra_arrivals;
+  int n_seqs, total_units;
+  int n_tokens[MD_MAX_BATCH];
+  int n_pages[MD_MAX_BATCH];
+  int chunks[MD_MAX_BATCH];
+  int unit_start[MD_MAX_BATCH + 1];
+};
+cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &tmap, int grid,
+                             cudaStream_t s);
+int attention_grid_limit(int ps);     // CTAs resident at once (0 on error)
+cudaError_t attention_prepare(int ps); // one-time function attributes
+
+/* --------------------------------------------------- fold / score ------- */
+struct ScoreParams {
+  const float *mass;
+  float *window, *a, *ahat, *prio, *page_score;
+  int32_t *t_ref;
+  const uint8_t *region;
+  const int32_t *block_table;
+  long long slots;
+  int rows, ps, P_max;
+  int fold_only;         // 1: window += mass rows and nothing else
+  int observe, mass_pending;
+  float norm;            // window steps * L * Hq
+  int t;
+  float rho, gamma, tau_scale, alpha;
+  int score_mode, page_reduce, keep_prio;
+  RegionTable reg;
+  int n_seqs, total_pages;
+  int n_tokens[MD_MAX_BATCH];
+  int n_pages[MD_MAX_BATCH];
+  int page_start[MD_MAX_BATCH + 1];
+};
+cudaError_t launch_score(const ScoreParams &p, cudaStream_t s);
+
+/* ------------------------------------------------------------- select --- */
+struct SelectParams {
+  const float *page_score;
+  int32_t *block_table;
+  int32_t *free_stack;
+  int32_t *evict_list;    // [max_batch][P_max] internal
+  int32_t *user_evicted;  // optional [n_seqs][P_max]
+  int *status;
+  int P_max, n_seqs, top;
+  int n_pages[MD_MAX_BATCH];
+  int n_evict[MD_MAX_BATCH];
+  int push_off[MD_MAX_BATCH];
+};
+cudaError_t launch_select(const SelectParams &p, cudaStream_t s);
+
+/* --------------------------------------------------------------- init --- */
+cudaError_t launch_init(int32_t *free_stack, int P_phys, int *status, int *counters,
+                        size_t n_items, cudaStream_t s);
+
+}  // namespace md
+
+#endif

@@ -1,0 +1,339 @@
+/* Stages 0, 2, 3, 4 of the MemDecay step and the workspace initialiser.
+ *
+ *   append   write new tokens' K/V into the page pool (taking fresh pages
+ *            from the free stack) and start each token's state: region label,
+ *            t_ref = insertion step, a = 0 (Sec. III-A; Fig. 1 "append KV").
+ *   score    per page, one lane per token: Abar from the window accumulator
+ *            and the per-(layer, KV head) mass rows (Sec. III-C), the EWMA
+ *            (Eq. 2), the refresh test Abar >= tau_scale/|K_t| (Eq. 3), the
+ *            retention score (Eq. 4, lambda = ln2 / half-life, Eq. 7) and the
+ *            page score by a shuffle reduction over the page's lanes (Eq. 5;
+ *            pinned pages and the page being written score +inf).  With
+ *            fold_only it only adds the mass rows into the window accumulator.
+ *   select   one CTA per sequence: radix select (4 passes of 8-bit digits
+ *            over order-preserving uint32 keys, ties by logical page index)
+ *            of the e lowest evictable pages, stable compaction of the block
+ *            table row, push of the freed ids onto the free stack
+ *            (Sec. III-D, Algorithm 1: lowest S_p first; a selection, not a
+ *            sort or a heap). */
+#include <float.h>
+
+#include "md_internal.h"
+#include "md_ptx.cuh"
+
+namespace md {
+
+/* ---------------------------------------------------------------- init --- */
+__global__ void init_kernel(int32_t *free_stack, int P_phys, int *status, int *counters,
+                            size_t n_items) {
+  const size_t stride = (size_t)gridDim.x * blockDim.x;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < (size_t)P_phys; i += stride)
+    free_stack[i] = P_phys - 1 - (int)i;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n_items; i += stride)
+    counters[i] = 0;
+  if (blockIdx.x == 0 && threadIdx.x < ST_WORDS) status[threadIdx.x] = 0;
+}
+
+cudaError_t launch_init(int32_t *free_stack, int P_phys, int *status, int *counters,
+                        size_t n_items, cudaStream_t s) {
+  init_kernel<<<304, 256, 0, s>>>(free_stack, P_phys, status, counters, n_items);
+  return cudaGetLastError();
+}
+
+/* -------------------------------------------------------------- append --- */
+/* One thread per 16-byte piece of a token's K or V row in one (layer, head). */
+__global__ void append_kernel(const __grid_constant__ AppendParams p) {
+  const long long per_token = (long long)p.L * p.Hkv * 2 * 16;
+  const long long total = (long long)p.n_seqs * p.n_per_seq * per_token;
+  for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
+       w += (long long)gridDim.x * blockDim.x) {
+    const int c = (int)(w & 15);
+    long long r = w >> 4;
+    const int kv = (int)(r & 1);
+    r >>= 1;
+    const int h = (int)(r % p.Hkv);
+    r /= p.Hkv;
+    const int l = (int)(r % p.L);
+    r /= p.L;
+    const int i = (int)(r % p.n_per_seq);
+    const int j = (int)(r / p.n_per_seq);
+    const int seq = p.seq0 + j;
+    const int tok = p.tok0[j] + i;
+    const int pg = tok / p.ps, off = tok - pg * p.ps;
+    const int pages_before = (p.tok0[j] + p.ps - 1) / p.ps;
+    int phys;
+    if (pg < pages_before)
+      phys = p.block_table[(size_t)seq * p.P_max + pg];
+    else
+      phys = p.free_stack[p.pop_base[j] - (pg - pages_before)];
+
+    const uint16_t *src = (kv == 0 ? p.k_src : p.v_src) + (long long)j * p.sb +
+                          (long long)l * p.sl + (long long)h * p.sh + (long long)i * p.si;
+    uint16_t *dst = p.pool +
+                    ((((size_t)l * p.P_phys + phys) * p.Hkv + h) * 2 + kv) * (size_t)p.ps * D +
+                    (size_t)off * D;
+    ((uint4 *)dst)[c] = ((const uint4 *)src)[c];
+
+    if (c == 0 && kv == 0 && h == 0 && l == 0) {
+      const size_t slot = (size_t)phys * p.ps + off;
+      p.region[slot] = p.regions_dev ? p.regions_dev[i] : p.regions_param[j];
+      p.t_ref[slot] = p.steps_dev ? p.steps_dev[i] : p.insert_step;
+      p.a[slot] = 0.f;
+      p.window[slot] = 0.f;
+      p.ahat[slot] = 0.f;
+      p.prio[slot] = 0.f;
+      if (off == 0 && pg >= pages_before) p.block_table[(size_t)seq * p.P_max + pg] = phys;
+    }
+  }
+}
+
+cudaError_t launch_append(const AppendParams &p, cudaStream_t s) {
+  const long long total = (long long)p.n_seqs * p.n_per_seq * p.L * p.Hkv * 32;
+  if (total == 0) return cudaSuccess;
+  long long blocks = (total + 255) / 256;
+  if (blocks > 152 * 16) blocks = 152 * 16;
+  append_kernel<<<(int)blocks, 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+/* ------------------------------------------------------ score / fold ----- */
+__device__ __forceinline__ int find_seq(const int *start, int n, int x) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (start[mid] <= x) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+/* Each warp handles 32/PS consecutive pages per iteration, one lane per
+ * token slot; the loop count is uniform across the warp so the segmented
+ * shuffle reductions see every lane. */
+template <int PS>
+__global__ void score_kernel(const __grid_constant__ ScoreParams p) {
+  constexpr int PPW = 32 / PS;
+  const int lane = threadIdx.x & 31;
+  const int warps_total = (gridDim.x * blockDim.x) >> 5;
+  const int warp_id = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const float INF = INFINITY;
+  for (int base = warp_id * PPW; base < p.total_pages; base += warps_total * PPW) {
+    const int gp = base + lane / PS;
+    const int off = lane % PS;
+    const bool page_ok = gp < p.total_pages;
+    int b = 0, pg = 0, P = 0;
+    bool valid = false;
+    size_t slot = 0;
+    if (page_ok) {
+      b = find_seq(p.page_start, p.n_seqs, gp);
+      pg = gp - p.page_start[b];
+      P = p.n_pages[b];
+      valid = pg * PS + off < p.n_tokens[b];
+      slot = (size_t)p.block_table[(size_t)b * p.P_max + pg] * PS + off;
+    }
+    float s = 0.f;
+    int pinned = 0;
+    if (valid) {
+      if (p.fold_only) {
+        float w = p.window[slot];
+        for (int r = 0; r < p.rows; ++r) w += p.mass[(size_t)r * p.slots + slot];
+        p.window[slot] = w;
+      } else {
+        const int reg = p.region[slot];
+        float a = p.a[slot];
+        int tr = p.t_ref[slot];
+        if (p.observe) {
+          float w = p.window[slot];
+          if (p.mass_pending)
+            for (int r = 0; r < p.rows; ++r) w += p.mass[(size_t)r * p.slots + slot];
+          const float abar = __fdiv_rn(w, p.norm);                    // Sec. III-C
+          a = p.rho * a + p.gamma * abar;                             // Eq. 2
+          const float tau = __fdiv_rn(p.tau_scale, (float)p.n_tokens[b]);
+          if (abar >= tau) tr = p.t;                                  // Eq. 3
+          p.window[slot] = 0.f;
+          p.ahat[slot] = abar;
+          p.a[slot] = a;
+          p.t_ref[slot] = tr;
+        }
+        const float x = __fdiv_rn((float)(p.t - tr), p.reg.half_life[reg]);
+        const float d = exp2f(-x);                                    // Eqs. 4, 7
+        s = (p.score_mode == 0) ? p.reg.base[reg] * d + p.alpha * a
+                                : (p.reg.base[reg] + p.alpha * a) * d;
+        pinned = p.reg.pinned[reg];
+        if (pinned) s = INF;
+        if (p.keep_prio) p.prio[slot] = s;
+      }
+    }
+    if (!p.fold_only) {
+      float sum = (valid && !pinned) ? s : 0.f;
+      float mx = (valid && !pinned) ? s : -INF;
+      int anyp = (valid && pinned) ? 1 : 0;
+      int cnt = valid ? 1 : 0;
+#pragma unroll
+      for (int o = PS / 2; o > 0; o >>= 1) {
+        sum += __shfl_xor_sync(0xffffffffu, sum, o, PS);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o, PS));
+        anyp |= __shfl_xor_sync(0xffffffffu, anyp, o, PS);
+        cnt += __shfl_xor_sync(0xffffffffu, cnt, o, PS);
+      }
+      if (page_ok && off == 0) {
+        float S;
+        if (anyp || pg == P - 1) S = INF;                            // pinning, tail
+        else S = (p.page_reduce == 0) ? __fdiv_rn(sum, (float)cnt) : mx;   // Eq. 5
+        p.page_score[(size_t)b * p.P_max + pg] = S;
+      }
+    }
+  }
+}
+
+cudaError_t launch_score(const ScoreParams &p, cudaStream_t s) {
+  if (p.total_pages == 0) return cudaSuccess;
+  const int ppb = 256 / p.ps;
+  long long blocks = (p.total_pages + ppb - 1) / ppb;
+  if (blocks > 152 * 8) blocks = 152 * 8;
+  if (p.ps == 16) score_kernel<16><<<(int)blocks, 256, 0, s>>>(p);
+  else score_kernel<32><<<(int)blocks, 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+/* -------------------------------------------------------------- select --- */
+constexpr int SEL_THREADS = 1024;
+constexpr uint32_t KEY_PINNED = 0xFFFFFFFFu;
+
+/* Order-preserving map of fp32 onto uint32 (larger float -> larger key). */
+__device__ __forceinline__ uint32_t order_key(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+/* Block-wide exclusive scan of one int per thread; returns the prefix and
+ * writes the block total to *total. */
+__device__ __forceinline__ int block_exclusive_scan(int v, int *warp_sums, int *total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    const int nw = blockDim.x >> 5;
+    int s = lane < nw ? warp_sums[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    if (lane < nw) warp_sums[lane] = s;   // inclusive sums of warps
+  }
+  __syncthreads();
+  const int before = (wid > 0 ? warp_sums[wid - 1] : 0) + x - v;
+  *total = warp_sums[(blockDim.x >> 5) - 1];
+  __syncthreads();
+  return before;
+}
+
+__global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_constant__ SelectParams p) {
+  extern __shared__ uint32_t sm[];
+  uint32_t *keys = sm;                               // [P_max]
+  int32_t *phys = (int32_t *)(sm + p.P_max);         // [P_max]
+  __shared__ int hist[256];
+  __shared__ int warp_sums[32];
+  __shared__ uint32_t s_prefix;
+  __shared__ int s_k, s_bad;
+
+  const int b = blockIdx.x;
+  const int P = p.n_pages[b];
+  const int e = p.n_evict[b];
+  int32_t *row = p.block_table + (size_t)b * p.P_max;
+  int32_t *uout = p.user_evicted ? p.user_evicted + (size_t)b * p.P_max : nullptr;
+  if (e == 0) {
+    if (uout)
+      for (int i = threadIdx.x; i < p.P_max; i += blockDim.x) uout[i] = -1;
+    return;
+  }
+  const float *sc = p.page_score + (size_t)b * p.P_max;
+  for (int i = threadIdx.x; i < P; i += blockDim.x) {
+    const float S = sc[i];
+    keys[i] = (S == INFINITY) ? KEY_PINNED : order_key(S);
+    phys[i] = row[i];
+  }
+  if (threadIdx.x == 0) { s_prefix = 0u; s_k = e; s_bad = 0; }
+  __syncthreads();
+
+  /* radix select of the e-th smallest evictable key, most significant digit first */
+  uint32_t mask = 0u;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    const uint32_t prefix = s_prefix;
+    for (int i = threadIdx.x; i < P; i += blockDim.x) {
+      const uint32_t k = keys[i];
+      if (k != KEY_PINNED && (k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int k = s_k, cum = 0, digit = -1;
+      for (int dgt = 0; dgt < 256; ++dgt) {
+        if (cum + hist[dgt] >= k) { digit = dgt; break; }
+        cum += hist[dgt];
+      }
+      if (digit < 0) s_bad = 1;           // fewer evictable pages than e
+      else { s_prefix = prefix | ((uint32_t)digit << shift); s_k = k - cum; }
+    }
+    __syncthreads();
+    if (s_bad) {
+      if (threadIdx.x == 0) atomicCAS(&p.status[ST_CODE], 0, (int)MD_ERR_STATE);
+      return;
+    }
+    mask |= 0xFFu << shift;
+  }
+  const uint32_t T = s_prefix;     // key of the e-th smallest evictable page
+  const int take_eq = s_k;         // how many pages with key == T are evicted
+
+  /* evict: key < T, or key == T among the first take_eq in logical order;
+   * compact kept pages in order; list the evicted ones in logical order */
+  int carry_eq = 0, carry_ev = 0;
+  const int base_push = p.top + p.push_off[b];
+  for (int t0 = 0; t0 < P; t0 += blockDim.x) {
+    const int i = t0 + threadIdx.x;
+    const bool in = i < P;
+    const uint32_t k = in ? keys[i] : KEY_PINNED;
+    const int eq = (in && k == T) ? 1 : 0;
+    int tot_eq;
+    const int rank_eq = carry_eq + block_exclusive_scan(eq, warp_sums, &tot_eq);
+    const int ev = (in && k != KEY_PINNED && (k < T || (eq && rank_eq < take_eq))) ? 1 : 0;
+    int tot_ev;
+    const int idx_ev = carry_ev + block_exclusive_scan(ev, warp_sums, &tot_ev);
+    if (in) {
+      const int id = phys[i];
+      if (ev) {
+        p.evict_list[(size_t)b * p.P_max + idx_ev] = id;
+        p.free_stack[base_push + idx_ev] = id;
+        if (uout) uout[idx_ev] = id;
+      } else {
+        row[i - idx_ev] = id;
+      }
+    }
+    carry_eq += tot_eq;
+    carry_ev += tot_ev;
+  }
+  __syncthreads();
+  for (int i = P - e + threadIdx.x; i < P; i += blockDim.x) row[i] = -1;
+  if (uout)
+    for (int i = e + threadIdx.x; i < p.P_max; i += blockDim.x) uout[i] = -1;
+}
+
+cudaError_t launch_select(const SelectParams &p, cudaStream_t s) {
+  if (p.n_seqs == 0) return cudaSuccess;
+  const size_t smem = (size_t)p.P_max * 8;
+  cudaError_t err = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+  if (err != cudaSuccess) return err;
+  select_kernel<<<p.n_seqs, SEL_THREADS, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace md

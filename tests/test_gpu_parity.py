@@ -1,0 +1,238 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the fp64
+oracle on the same seeded inputs (tolerances in tests/gpu_harness.py)."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # pragma: no cover - GPU tests only run on the GPU machine
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import paper_2607_10582_gb300 as md  # noqa: E402
+import synth  # noqa: E402
+from paper_2607_10582_gb300 import build as mdbuild  # noqa: E402
+from tests.gpu_harness import Lockstep, to_dev  # noqa: E402
+
+mdbuild.build()
+synth.build()
+
+
+def test_cuda_generator_matches_host():
+    regions = (np.arange(300) % 7).astype(np.uint8)
+    for structured in (False, True):
+        k, v = synth.kv_host(5, 3, 2, 2, 40, 300, regions, structured)
+        kd = torch.empty(k.shape, dtype=torch.int16, device="cuda")
+        vd = torch.empty(v.shape, dtype=torch.int16, device="cuda")
+        rd = torch.from_numpy(regions).cuda()
+        kap = (synth.ctypes.c_float * 9)(*synth.KAPPA_STRUCT) if structured else None
+        assert synth.lib().synth_fill_kv_dev(5, int(structured), kap, 3, 2, 2, 128, 40, 300,
+                                             rd.data_ptr(), kd.data_ptr(), vd.data_ptr(), None) == 0
+        torch.cuda.synchronize()
+        assert np.array_equal(kd.cpu().numpy().view(np.uint16), k)
+        assert np.array_equal(vd.cpu().numpy().view(np.uint16), v)
+    q = synth.q_host(9, 3, 2, 12, 2, 11, True)
+    qd = torch.empty(q.shape, dtype=torch.int16, device="cuda")
+    kap = (synth.ctypes.c_float * 9)(*synth.KAPPA_STRUCT)
+    assert synth.lib().synth_fill_q_dev(9, 1, kap, 3, 2, 12, 6, 128, 11, qd.data_ptr(), None) == 0
+    torch.cuda.synchronize()
+    assert np.array_equal(qd.cpu().numpy().view(np.uint16), q)
+
+
+def test_config0_full_run():
+    """Config 0 end to end: 448-token trace, 64 decode steps, eviction to 50%
+    of pages at every step."""
+    ls = Lockstep(synth.make_workload(0)).run()
+    ls.check_layout()
+    assert ls.max_err["O"] < 2e-2
+
+
+def test_multichunk_ragged_batch():
+    """Ragged sequences long enough to split each (layer, head) item into many
+    chunks, GQA group 8, pages of 16 with partial last pages."""
+    w = synth.custom_workload("ragged", L=2, Hq=16, Hkv=2, page_size=16,
+                              lengths=[37, 1300, 5003], budget_frac=0.4, steps=12, seed=3)
+    ls = Lockstep(w).run()
+    ls.check_layout()
+
+
+def test_group6_page32_structured():
+    """Group of 6 query heads (padded to 8 in the kernel), pages of 32, keys
+    and queries with region structure and hot tokens so refreshes fire."""
+    w = synth.custom_workload("g6", L=3, Hq=12, Hkv=2, page_size=32, lengths=[700, 2100],
+                              budget_frac=0.5, steps=12, seed=4, structured=True)
+    ls = Lockstep(w).run()
+    ls.check_layout()
+
+
+def test_observation_window():
+    """Observation every 4 decode steps: the mass of the window's steps is
+    accumulated and averaged (Sec. III-C)."""
+    w = synth.custom_workload("win", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900, 600],
+                              budget_frac=0.5, steps=16, seed=5, window_k=4, structured=True)
+    ls = Lockstep(w).run()
+    ls.check_layout()
+
+
+@pytest.mark.parametrize("score_mode,page_reduce,w", [(1, 0, 4.0), (0, 1, 0.5), (1, 1, 0.0)])
+def test_score_variants(score_mode, page_reduce, w):
+    wl = synth.custom_workload("var", L=2, Hq=16, Hkv=2, page_size=16, lengths=[800, 1000],
+                               budget_frac=0.3, steps=8, seed=6, score_mode=score_mode,
+                               page_reduce=page_reduce, attn_weight=w, structured=True)
+    Lockstep(wl).run().check_layout()
+
+
+def test_pins_over_budget_warns():
+    """Pinned pages alone exceed the budget: every evictable page goes, the
+    warning comes back, pinned pages stay."""
+    w = synth.custom_workload("pins", L=1, Hq=8, Hkv=2, page_size=16, lengths=[400],
+                              budget_frac=0.1, steps=2, seed=7)
+    w.regions[0][:] = synth.SYSTEM
+    w.regions[0][100:180] = synth.TOOL_OUT
+    ls = Lockstep(w)
+    ls.prefill()
+    ls.decode()
+    n = ls.observe()
+    assert n[0] > 0
+    st, _ = ls.gpu.evict([1])
+    assert st == md.MD_WARN_OVER_BUDGET
+
+
+def test_config1_first_steps():
+    """Config 1 geometry (Qwen2.5-1.5B, 28 layers, 12/2 heads), 1,700 tokens."""
+    ls = Lockstep(synth.make_workload(1))
+    ls.run(steps=20)
+    ls.check_layout()
+
+
+def test_config2_first_steps():
+    """Config 2 geometry (Qwen2.5-3B, 36 layers, 16/2), 32 sequences with
+    Dirichlet region spans and insertion offsets."""
+    ls = Lockstep(synth.make_workload(2))
+    ls.run(steps=3)
+    ls.check_layout()
+
+
+def _small_run(seed):
+    w = synth.custom_workload("det", L=2, Hq=16, Hkv=2, page_size=16, lengths=[700, 1500],
+                              budget_frac=0.5, steps=6, seed=seed, structured=True)
+    c = md.Cache(w.L, w.Hq, w.Hkv, w.page_size, w.B, w.max_pages_per_seq(), w.num_phys_pages())
+    for r in range(7):
+        c.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    for b in range(w.B):
+        k, v = synth.kv_host(w.seed, b, w.L, w.Hkv, 0, w.n0(b), w.regions[b], True)
+        c.append_tokens(b, w.regions[b], to_dev(k), to_dev(v))
+    outs = []
+    pos = [w.n0(b) for b in range(w.B)]
+    for t in range(1, 7):
+        q = synth.q_host(w.seed, w.B, w.L, w.Hq, w.Hkv, t, True)
+        kn, vn = synth.step_kv_host(w.seed, pos, [6] * w.B, w.L, w.Hkv, True)
+        out = torch.empty((w.B, w.L, w.Hq, 128), dtype=torch.int16, device="cuda")
+        c.decode_step(w.B, to_dev(q), to_dev(kn), to_dev(vn), [6] * w.B, out)
+        c.evict(w.budget_pages)
+        pos = [p + 1 for p in pos]
+        outs.append(out.clone())
+    states = [c.get_state(s) for s in (md.MD_STATE_A, md.MD_STATE_AHAT, md.MD_STATE_PAGE_SCORE,
+                                       md.MD_STATE_BLOCK_TABLE, md.MD_STATE_FREE)]
+    torch.cuda.synchronize()
+    return outs, states
+
+
+def test_bit_identical_reruns():
+    """No float atomics anywhere: two runs give bit-identical outputs and
+    state (a proxy for the absence of races)."""
+    o1, s1 = _small_run(8)
+    o2, s2 = _small_run(8)
+    for x, y in zip(o1 + s1, o2 + s2):
+        assert torch.equal(x, y)
+
+
+def test_checkpoint_restore_replays_step():
+    w = synth.custom_workload("ckpt", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900],
+                              budget_frac=0.3, steps=2, seed=9)
+    ls = Lockstep(w)
+    ls.prefill()
+    ls.decode()
+    ls.observe()
+    saved = ls.gpu.save_state()
+    q = synth.q_host(w.seed, 1, w.L, w.Hq, w.Hkv, 99)
+    kn, vn = synth.step_kv_host(w.seed, [5000], [6], w.L, w.Hkv)
+    res = []
+    for _ in range(2):
+        ls.gpu.load_state(saved)
+        out = torch.empty((1, w.L, w.Hq, 128), dtype=torch.int16, device="cuda")
+        ls.gpu.decode_step(1, to_dev(q), to_dev(kn), to_dev(vn), [6], out)
+        ls.gpu.evict([3])
+        res.append((out.clone(), ls.gpu.get_state(md.MD_STATE_BLOCK_TABLE),
+                    ls.gpu.get_state(md.MD_STATE_PAGE_SCORE)))
+    torch.cuda.synchronize()
+    for x, y in zip(res[0], res[1]):
+        assert torch.equal(x, y)
+
+
+def test_capacity_and_argument_errors_are_synchronous():
+    c = md.Cache(1, 8, 2, 16, 2, 4, 6)
+    k = torch.zeros((1, 2, 80, 128), dtype=torch.int16, device="cuda")
+    with pytest.raises(md.MemDecayError) as e:
+        c.append_tokens(0, np.zeros(80, np.uint8), k, k)          # 5 pages > 4
+    assert e.value.status == md.MD_ERR_CAPACITY
+    assert c.query(md.MD_QUERY_TOKENS, 0) == 0 and c.query(md.MD_QUERY_FREE_TOP) == 6
+    with pytest.raises(md.MemDecayError) as e:
+        c.append_tokens(0, np.full(3, 9, np.uint8), k[:, :, :3].contiguous(), k[:, :, :3].contiguous())
+    assert e.value.status == md.MD_ERR_INVALID_ARG
+    with pytest.raises(md.MemDecayError) as e:
+        c.append_tokens(0, np.zeros(3, np.uint8), k, k, insert_steps=[0, 1, 5])
+    assert e.value.status == md.MD_ERR_INVALID_ARG
+    with pytest.raises(md.MemDecayError) as e:
+        c.set_region_params(1, 1.0, 0.0, False)
+    assert e.value.status == md.MD_ERR_INVALID_ARG
+    c.append_tokens(0, np.zeros(3, np.uint8), k[:, :, :3].contiguous(), k[:, :, :3].contiguous())
+    with pytest.raises(md.MemDecayError) as e:
+        c.set_region_params(0, 1.0, 10.0, True)   # pinned flag with tokens cached
+    assert e.value.status == md.MD_ERR_STATE
+    assert c.sync() == md.MD_OK
+
+
+def test_single_token_and_no_eviction_edges():
+    """One cached token (o = v exactly, Abar = 1), and budgets at or above
+    the page count (nothing evicted)."""
+    w = synth.custom_workload("tiny", L=1, Hq=8, Hkv=2, page_size=16, lengths=[0],
+                              budget_frac=1.0, steps=1, seed=10)
+    ls = Lockstep(w)
+    ls.decode()
+    n = ls.observe(budgets=[5])
+    assert list(n) == [0]
+    ah = ls.gpu.get_state(md.MD_STATE_AHAT).cpu().numpy()
+    slot = ls.orc.slots(0)[0]
+    assert abs(ah[slot] - 1.0) < 1e-6
+    for _ in range(40):
+        ls.decode()
+        ls.observe(budgets=[100])
+    ls.check_layout()
+
+
+def test_device_wait_timeout_is_reported_not_hung():
+    """An exchange wait that nothing completes (an injected extra arrival)
+    runs out after its bounded spin; the kernel records the timeout and
+    returns; the CUDA context stays usable and the handle refuses more work."""
+    w = synth.custom_workload("to", L=1, Hq=8, Hkv=2, page_size=16, lengths=[600],
+                              budget_frac=0.5, steps=1, seed=11)
+    ls = Lockstep(w)
+    ls.prefill()
+    ls.gpu.debug_set(md.MD_DEBUG_SPIN_LIMIT_NS, 20_000_000)
+    ls.gpu.debug_set(md.MD_DEBUG_EXTRA_ARRIVALS, 1)
+    q = synth.q_host(w.seed, 1, 1, 8, 2, 1)
+    kn, vn = synth.step_kv_host(w.seed, [600], [6], 1, 2)
+    out = torch.empty((1, 1, 8, 128), dtype=torch.int16, device="cuda")
+    ls.gpu.decode_step(1, to_dev(q), to_dev(kn), to_dev(vn), [6], out)
+    assert ls.gpu.sync() == md.MD_ERR_DEVICE_TIMEOUT
+    with pytest.raises(md.MemDecayError) as e:
+        ls.gpu.evict([2])
+    assert e.value.status == md.MD_ERR_STATE
+    x = torch.arange(10, device="cuda").sum()
+    assert int(x) == 45
+    ls2 = Lockstep(w)
+    ls2.prefill()
+    ls2.decode()
+    ls2.observe()

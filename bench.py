@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--w", type=float, default=1.0, help="attention weight (config 4 sweeps 0/0.5/1/4)")
     ap.add_argument("--phase", default="full", choices=["full", "steady"])
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--max-tokens", type=int, default=0,
+                    help="truncate every trace to this many tokens (small profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -159,8 +161,7 @@ def run_native(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     stream = torch.cuda.current_stream(dev)
-    over = {"attn_weight": args.w} if args.config == 4 else {}
-    w = synth.make_workload(args.config, seed=args.seed + rank, **over)
+    w = make_workload(args, args.seed + rank)
     B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
     cache = md.Cache(L, Hq, Hkv, ps, B, w.max_pages_per_seq(), w.num_phys_pages(),
                      rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
@@ -319,10 +320,20 @@ def cpu_cores_used():
     return 1
 
 
-def run_reference(args):
+def make_workload(args, seed):
     import synth
     over = {"attn_weight": args.w} if args.config == 4 else {}
-    w = synth.make_workload(args.config, seed=args.seed, **over)
+    w = synth.make_workload(args.config, seed=seed, **over)
+    if args.max_tokens:
+        n = args.max_tokens
+        w.regions = [r[:n].copy() for r in w.regions]
+        w.insert_steps = [s[:n].copy() for s in w.insert_steps]
+        w.name += f" (traces truncated to {n} tokens)"
+    return w
+
+
+def run_reference(args):
+    w = make_workload(args, args.seed)
     layers = 1
     o0, inputs = oracle_sample(w, layers)
     tokens_step = sum(w.n0(b) + 1 for b in range(w.B))

@@ -40,13 +40,16 @@ struct AttnShape {
   static constexpr int NT = PS / 16;                 // 16-token tiles per page
   static constexpr int HALF_BYTES = 2 * PS * 128;    // 64 columns of K and V rows
   static constexpr int STAGE_BYTES = 2 * HALF_BYTES; // one page of one (layer, KV head)
-  static constexpr int R = (PS == 16) ? 16 : 8;      // ring stages (128 KiB)
+  static constexpr int R = (PS == 16) ? 8 : 4;       // ring stages (64 KiB per CTA)
   static constexpr int RING_BYTES = R * STAGE_BYTES;
+  static constexpr int CTAS_PER_SM = 2;
   static constexpr int THREADS = 32 * (NCW + 1);
-  static constexpr int MERGE_FLOATS = NCW * (16 + GP * D);
-  static constexpr int FIN_FLOATS = 16 + MD_MAX_CHUNKS * GP;
-  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * R * 8 + 4 * MERGE_FLOATS +
-                                 4 * FIN_FLOATS + 64;
+  static constexpr int Q_BYTES = GP * D * 2;         // one unit's query heads
+  static constexpr int MAX_UNIT_PAGES = MD_MAX_CHUNK_TOKENS / PS;
+  static constexpr int MERGE_FLOATS = NCW * (24 + GP * D);
+  static constexpr int FIN_FLOATS = 16 + 3 * MD_MAX_CHUNKS * GP;
+  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * Q_BYTES + (2 * R + 4) * 8 +
+                                 4 * MERGE_FLOATS + 4 * FIN_FLOATS + 4 * MAX_UNIT_PAGES + 64;
 };
 
 struct Unit {
@@ -105,30 +108,43 @@ __device__ __forceinline__ uint32_t swz(uint32_t stage, int row, int d) {
 }
 
 template <int PS, int NCW>
-__global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
+__global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW>::CTAS_PER_SM)
     attn_mass_kernel(const __grid_constant__ AttnParams p,
                      const __grid_constant__ CUtensorMap tmap) {
   using S = AttnShape<PS, NCW>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t *ring = smem;
-  uint64_t *full = (uint64_t *)(ring + S::RING_BYTES);
+  uint8_t *sQ = ring + S::RING_BYTES;                   // [2][8 heads][128] bf16
+  uint64_t *full = (uint64_t *)(sQ + 2 * S::Q_BYTES);
   uint64_t *empty = full + S::R;
-  float *wm = (float *)(empty + S::R);        // [NCW][8] per-warp running max
+  uint64_t *qfull = empty + S::R;                       // [2]
+  uint64_t *qempty = qfull + 2;                         // [2]
+  float *wm = (float *)(qempty + 2);          // [NCW][8] per-warp running max
   float *wl = wm + NCW * 8;                   // [NCW][8] per-warp running sum
-  float *wO = wl + NCW * 8;                   // [NCW][8][128] per-warp O^T
-  float *fin = wm + S::MERGE_FLOATS;          // [16]: unit max m[8] then 8 spare
-  float *fac = fin + 16;                      // [MD_MAX_CHUNKS][8] combine factors
-  int *flag = (int *)(fac + MD_MAX_CHUNKS * GP);
+  float *wf = wl + NCW * 8;                   // [NCW][8] per-warp merge factor
+  float *wO = wf + NCW * 8;                   // [NCW][8][128] per-warp O^T
+  float *fin = wm + S::MERGE_FLOATS;          // [16]: head max, then 1/Z
+  float *pm = fin + 16;                       // [MD_MAX_CHUNKS][8] partial maxima
+  float *pl = pm + MD_MAX_CHUNKS * GP;        // [MD_MAX_CHUNKS][8] partial sums
+  float *fac = pl + MD_MAX_CHUNKS * GP;       // [MD_MAX_CHUNKS][8] combine factors
+  int *sphys = (int *)(fac + MD_MAX_CHUNKS * GP);   // [MAX_UNIT_PAGES] page ids
+  int *flag = sphys + S::MAX_UNIT_PAGES;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const uint32_t ring_u32 = smem_u32(ring);
+  const uint32_t sQ_u32 = smem_u32(sQ);
+  const int G = p.G;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S::R; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(smem_u32(&qfull[s]), 1);
+      mbar_init(smem_u32(&qempty[s]), NCW);
     }
     flag[0] = flag[1] = flag[2] = 0;
     fence_barrier_init();
@@ -140,10 +156,20 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       tma_prefetch_desc(&tmap);
-      int i = 0;
+      int i = 0, nu = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x, ++nu) {
         const Unit un = decode_unit(p, u);
+        /* the unit's G query rows: one bulk copy into a double-buffered slot */
+        const int qs = nu & 1;
+        if (nu >= 2 && !wait_phase(smem_u32(&qempty[qs]), ((nu >> 1) - 1) & 1, p, 5, true)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(smem_u32(&qfull[qs]), G * D * 2);
+        bulk_load(sQ_u32 + qs * S::Q_BYTES,
+                  p.q + (((size_t)un.b * p.L + un.l) * p.Hq + (size_t)un.kvh * G) * D, G * D * 2,
+                  smem_u32(&qfull[qs]));
         const int32_t *bt = p.block_table + (size_t)un.b * p.P_max;
         for (int pg = un.p0; pg < un.p1; ++pg, ++i) {
           const int s = i % S::R;
@@ -159,10 +185,13 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
           tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
           tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
         }
+        if (!ok) { ++nu; break; }
       }
       /* No copy may still be writing this CTA's shared memory when it exits. */
       for (int k = (i > S::R ? i - S::R : 0); k < i; ++k)
         wait_phase(smem_u32(&full[k % S::R]), (k / S::R) & 1, p, 2, false);
+      for (int k = (nu > 2 ? nu - 2 : 0); k < nu; ++k)
+        wait_phase(smem_u32(&qfull[k & 1]), (k >> 1) & 1, p, 6, false);
     }
     return;
   }
@@ -172,7 +201,6 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
   const int ct = threadIdx.x - 32;
   const int NC = NCW * 32;
   const int g = lane >> 2, t = lane & 3;
-  const int G = p.G;
   const bool hv0 = (2 * t) < G, hv1 = (2 * t + 1) < G;
   const uint64_t pol_keep = policy_evict_last();
   const float NEG_INF = -INFINITY;
@@ -183,8 +211,9 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
   bool aborted = false;   // this warp gave up a wait
   bool stopped = false;   // all consumer warps leave the unit loop together
 
+  /* Deferred end of a unit: wait for the item's other chunks, combine the
+   * partials (this chunk's slice of O), turn the stored scores into masses. */
   auto finish = [&](const Unit &pv, int pv_slot) -> bool {
-    /* wait until every chunk of the item published its partial */
     if (ct == 0) {
       const int target = pv.C + p.extra_arrivals;
       int okw = 1;
@@ -197,60 +226,91 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
             okw = 0;
             break;
           }
-          __nanosleep(100);
+          __nanosleep(64);
         }
       }
       flag[2] = okw ? 0 : 1;
     }
     named_barrier(1, NC);
     if (flag[2]) return false;
+    const int C = pv.C;
     const float *base = p.partials + (size_t)pv.X * p.chunk_stride * PARTIAL_FLOATS;
-    if (ct < GP) {
+    const int32_t *bt = p.block_table + (size_t)pv.b * p.P_max;
+    for (int idx = ct; idx < C * GP; idx += NC) {
+      const float *pj = base + (size_t)(idx >> 3) * PARTIAL_FLOATS;
+      pm[idx] = __ldcg(pj + (idx & 7));
+      pl[idx] = __ldcg(pj + 8 + (idx & 7));
+    }
+    for (int k = ct; k < pv.p1 - pv.p0; k += NC) sphys[k] = bt[pv.p0 + k];
+    named_barrier(1, NC);
+    if (cw == 0) {
+      /* per head: global max and normaliser over the C chunks */
+      const int h = lane & 7, part = lane >> 3;
       float M = NEG_INF;
-      for (int j = 0; j < pv.C; ++j) M = fmaxf(M, __ldcg(base + (size_t)j * PARTIAL_FLOATS + ct));
+      for (int j = part; j < C; j += 4) M = fmaxf(M, pm[j * GP + h]);
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 8));
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 16));
       const float Mr = (M == NEG_INF) ? 0.f : M;
       float Z = 0.f;
-      for (int j = 0; j < pv.C; ++j) {
-        const float *pj = base + (size_t)j * PARTIAL_FLOATS;
-        Z += exp2f(__ldcg(pj + ct) - Mr) * __ldcg(pj + 8 + ct);
+      for (int j = part; j < C; j += 4) Z += exp2f(pm[j * GP + h] - Mr) * pl[j * GP + h];
+      Z += __shfl_xor_sync(0xffffffffu, Z, 8);
+      Z += __shfl_xor_sync(0xffffffffu, Z, 16);
+      if (part == 0) {
+        fin[h] = Mr;
+        fin[8 + h] = Z > 0.f ? 1.f / Z : 0.f;
       }
-      const float invZ = Z > 0.f ? 1.f / Z : 0.f;
-      fin[ct] = Mr;
-      fin[8 + ct] = invZ;
-      for (int j = 0; j < pv.C; ++j)
-        fac[j * GP + ct] = exp2f(__ldcg(base + (size_t)j * PARTIAL_FLOATS + ct) - Mr) * invZ;
     }
     named_barrier(1, NC);
-    /* this chunk's slice of the item's output O[h][d], h < G */
-    const int E = G * D;
-    const int lo = (int)(((long long)pv.j * E) / pv.C);
-    const int hi = (int)(((long long)(pv.j + 1) * E) / pv.C);
-    uint16_t *orow = p.out + (((size_t)pv.b * p.L + pv.l) * p.Hq + (size_t)pv.kvh * G) * D;
-    for (int e = lo + ct; e < hi; e += NC) {
-      const int h = e >> 7;
-      float acc = 0.f;
-      for (int j = 0; j < pv.C; ++j)
-        acc += fac[j * GP + h] * __ldcg(base + (size_t)j * PARTIAL_FLOATS + 16 + e);
-      __nv_bfloat16 v = __float2bfloat16_rn(acc);
-      orow[e] = *(uint16_t *)&v;
+    for (int idx = ct; idx < C * GP; idx += NC)
+      fac[idx] = exp2f(pm[idx] - fin[idx & 7]) * fin[8 + (idx & 7)];
+    named_barrier(1, NC);
+    /* this chunk's slice of the item's output O[h][d] (h < G): four threads
+     * per element, each summing a quarter of the chunks */
+    {
+      const int E = G * D;
+      const int lo = (int)(((long long)pv.j * E) / C);
+      const int hi = (int)(((long long)(pv.j + 1) * E) / C);
+      uint16_t *orow = p.out + (((size_t)pv.b * p.L + pv.l) * p.Hq + (size_t)pv.kvh * G) * D;
+      const int q4 = ct & 3;
+      for (int e0 = lo; e0 < hi; e0 += NC / 4) {
+        const int e = e0 + (ct >> 2);
+        float acc = 0.f;
+        if (e < hi) {
+          const int h = e >> 7;
+#pragma unroll 4
+          for (int j = q4; j < C; j += 4)
+            acc += fac[j * GP + h] * __ldcg(base + (size_t)j * PARTIAL_FLOATS + 16 + e);
+        }
+        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+        if (q4 == 0 && e < hi) {
+          __nv_bfloat16 v = __float2bfloat16_rn(acc);
+          orow[e] = *(uint16_t *)&v;
+        }
+      }
     }
     /* token masses of this chunk from its stored scores */
-    const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + pv_slot) * p.scratch_tokens * GP;
-    const int ntok = (pv.p1 - pv.p0) * PS;
-    const int nvalid = p.n_tokens[pv.b] - pv.p0 * PS;
-    const int32_t *bt = p.block_table + (size_t)pv.b * p.P_max;
-    float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
-    for (int tk = ct; tk < ntok; tk += NC) {
-      if (tk >= nvalid) continue;
-      const float4 s0 = *(const float4 *)(scr + (size_t)tk * GP);
-      const float4 s1 = *(const float4 *)(scr + (size_t)tk * GP + 4);
-      const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-      float m = 0.f;
+    {
+      const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + pv_slot) * p.scratch_tokens * GP;
+      const int ntok = (pv.p1 - pv.p0) * PS;
+      const int nvalid = min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
+      float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
+      float fm[GP], fz[GP];
 #pragma unroll
-      for (int h = 0; h < GP; ++h)
-        if (h < G) m += exp2f(sv[h] - fin[h]) * fin[8 + h];
-      const int pg = pv.p0 + tk / PS;
-      mrow[(size_t)bt[pg] * PS + (tk % PS)] = m;
+      for (int h = 0; h < GP; ++h) {
+        fm[h] = fin[h];
+        fz[h] = (h < G) ? fin[8 + h] : 0.f;
+      }
+#pragma unroll 4
+      for (int tk = ct; tk < nvalid; tk += NC) {
+        const float4 s0 = __ldcg((const float4 *)(scr + (size_t)tk * GP));
+        const float4 s1 = __ldcg((const float4 *)(scr + (size_t)tk * GP + 4));
+        float m = exp2f(s0.x - fm[0]) * fz[0] + exp2f(s0.y - fm[1]) * fz[1] +
+                  exp2f(s0.z - fm[2]) * fz[2] + exp2f(s0.w - fm[3]) * fz[3];
+        m += exp2f(s1.x - fm[4]) * fz[4] + exp2f(s1.y - fm[5]) * fz[5] +
+             exp2f(s1.z - fm[6]) * fz[6] + exp2f(s1.w - fm[7]) * fz[7];
+        mrow[(size_t)sphys[tk / PS] * PS + (tk % PS)] = m;
+      }
     }
     named_barrier(1, NC);
     if (ct == 0) {
@@ -266,17 +326,26 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
     const int slot = nunit & 1;
     float *scr = p.scratch + ((size_t)blockIdx.x * 2 + slot) * p.scratch_tokens * GP;
 
-    /* Q^T fragments (B operand): head g, dims 16kk + {2t, 2t+1, 2t+8, 2t+9} */
+    /* Q^T fragments (B operand) from the prefetched rows: head g, dims
+     * 16kk + {2t, 2t+1} and 16kk + 8 + {2t, 2t+1}; padded heads are zero. */
     uint32_t qf[8][2];
     {
-      const uint16_t *qrow =
-          p.q + (((size_t)un.b * p.L + un.l) * p.Hq + (size_t)un.kvh * G + g) * D;
-      const bool gv = g < G;
+      const int qs = nunit & 1;
+      if (!wait_phase(smem_u32(&qfull[qs]), (nunit >> 1) & 1, p, 7, true)) aborted = true;
+      const int mi = lane >> 3, rr = lane & 7;
+      const uint32_t qb = sQ_u32 + qs * S::Q_BYTES + rr * (D * 2) + mi * 16;
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        qf[kk][0] = gv ? *(const uint32_t *)(qrow + 16 * kk + 2 * t) : 0u;
-        qf[kk][1] = gv ? *(const uint32_t *)(qrow + 16 * kk + 8 + 2 * t) : 0u;
+      for (int kk = 0; kk < 8; kk += 2) {
+        uint32_t r0, r1, r2, r3;
+        ldmatrix_x4(qb + kk * 32, r0, r1, r2, r3);
+        const bool gv = g < G;
+        qf[kk][0] = gv ? r0 : 0u;
+        qf[kk][1] = gv ? r1 : 0u;
+        qf[kk + 1][0] = gv ? r2 : 0u;
+        qf[kk + 1][1] = gv ? r3 : 0u;
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&qempty[qs]));
     }
     float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
     float o[8][4];
@@ -394,8 +463,11 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
       for (int w = 0; w < NCW; ++w) M = fmaxf(M, wm[w * 8 + ct]);
       const float Mr = (M == NEG_INF) ? 0.f : M;
       float Lsum = 0.f;
-      for (int w = 0; w < NCW; ++w) Lsum += exp2f(wm[w * 8 + ct] - Mr) * wl[w * 8 + ct];
-      fin[ct] = Mr;
+      for (int w = 0; w < NCW; ++w) {
+        const float f = exp2f(wm[w * 8 + ct] - Mr);
+        wf[w * 8 + ct] = f;
+        Lsum += f * wl[w * 8 + ct];
+      }
       part[ct] = M;
       part[8 + ct] = Lsum;
     }
@@ -403,7 +475,8 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, 1)
     for (int e = ct; e < GP * D; e += NC) {
       const int h = e >> 7;
       float acc = 0.f;
-      for (int w = 0; w < NCW; ++w) acc += exp2f(wm[w * 8 + h] - fin[h]) * wO[(size_t)w * GP * D + e];
+#pragma unroll
+      for (int w = 0; w < NCW; ++w) acc += wf[w * 8 + h] * wO[(size_t)w * GP * D + e];
       part[16 + e] = acc;
     }
     __threadfence();

@@ -1,0 +1,146 @@
+"""Full-size parity at configs 3 and 4, in the benchmark's launch
+configuration (the whole batch, 77 GB of K/V per step, on the GPU), checked
+on sampled sequences that the oracle recomputes one by one.
+
+Sequences are independent in every stage except the shared page pool, so the
+oracle runs a sampled sequence alone (its physical page ids differ) and the
+comparison is by logical token / logical page: attention output, Abar, a,
+clocks, token and page priorities, the evicted logical pages and the order of
+the compacted block-table row.  Tolerances as in tests/gpu_harness.py."""
+import gc
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+if not torch.cuda.is_available():  # pragma: no cover
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import oracle.memdecay_oracle as om  # noqa: E402
+import paper_2607_10582_gb300 as md  # noqa: E402
+import synth  # noqa: E402
+from paper_2607_10582_gb300 import build as mdbuild  # noqa: E402
+from tests.gpu_harness import TIE_REL, TOL_FLOOR, TOL_O_ABS, TOL_REL, rel_err  # noqa: E402
+
+mdbuild.build()
+synth.build()
+
+
+def gpu_run(w, steps):
+    """Prefill the whole batch with the CUDA generator, run `steps` decode
+    steps and one observation; return the GPU state needed for comparison."""
+    dev = torch.device("cuda")
+    B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
+    cache = md.Cache(L, Hq, Hkv, ps, B, w.max_pages_per_seq(), w.num_phys_pages(),
+                     rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
+                     score_mode=w.score_mode, page_reduce=w.page_reduce)
+    for r in range(7):
+        cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    lib = synth.lib()
+    nmax = max(w.n0(b) for b in range(B))
+    kb = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
+    vb = torch.empty_like(kb)
+    for b in range(B):
+        rd = torch.from_numpy(w.regions[b]).to(dev)
+        assert lib.synth_fill_kv_dev(w.seed, 0, None, b, L, Hkv, D, 0, w.n0(b), rd.data_ptr(),
+                                     kb.data_ptr(), vb.data_ptr(), None) == 0
+        cache.append_tokens(b, w.regions[b], kb.data_ptr(), vb.data_ptr(), w.insert_steps[b])
+        torch.cuda.synchronize()
+    del kb, vb
+    q = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((B, L, Hkv, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    outs = []
+    regs = [w.decode_region] * B
+    rdev = torch.tensor(regs, dtype=torch.uint8, device=dev)
+    for t in range(1, steps + 1):
+        pos = torch.tensor([w.n0(b) + t - 1 for b in range(B)], dtype=torch.int32, device=dev)
+        assert lib.synth_fill_q_dev(w.seed, 0, None, B, L, Hq, Hq // Hkv, D, t, q.data_ptr(), None) == 0
+        assert lib.synth_fill_step_kv_dev(w.seed, 0, None, B, L, Hkv, D, pos.data_ptr(), rdev.data_ptr(),
+                                          kn.data_ptr(), vn.data_ptr(), None) == 0
+        out = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+        cache.decode_step(B, q, kn, vn, regs, out)
+        outs.append(out)
+    pre_bt = cache.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
+    pre_tokens = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+    st, n_ev = cache.evict(w.budget_pages)
+    torch.cuda.synchronize()
+    assert cache.sync() == md.MD_OK
+    res = dict(st=st, n_ev=n_ev, pre_bt=pre_bt, pre_tokens=pre_tokens,
+               outs=[o.cpu().numpy().view(np.uint16) for o in (outs[0], outs[-1])])
+    for name, what in (("ahat", md.MD_STATE_AHAT), ("a", md.MD_STATE_A), ("t_ref", md.MD_STATE_T_REF),
+                       ("prio", md.MD_STATE_TOKEN_PRIO), ("page", md.MD_STATE_PAGE_SCORE),
+                       ("bt", md.MD_STATE_BLOCK_TABLE)):
+        res[name] = cache.get_state(what).cpu().numpy()
+    cache.close()
+    del cache, outs, q, kn, vn
+    gc.collect()
+    torch.cuda.empty_cache()
+    return res
+
+
+def oracle_run(w, b, steps):
+    """The oracle for sequence b alone, same inputs, same schedule."""
+    n = w.n0(b)
+    P0 = w.pages0(b)
+    cfg = om.OracleConfig(w.L, w.Hq, w.Hkv, w.D, w.page_size, 1, w.max_pages_per_seq(),
+                          P0 + steps // w.page_size + 2, rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale,
+                          attn_weight=w.attn_weight, score_mode=w.score_mode, page_reduce=w.page_reduce)
+    o = om.Oracle(cfg)
+    for r in range(7):
+        o.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    k, v = synth.kv_host(w.seed, b, w.L, w.Hkv, 0, n, w.regions[b])
+    o.append_tokens(0, w.regions[b], k, v, w.insert_steps[b])
+    del k, v
+    outs = []
+    for t in range(1, steps + 1):
+        q = synth.q_host(w.seed, w.B, w.L, w.Hq, w.Hkv, t)[b:b + 1]
+        kn, vn = synth.kv_host(w.seed, b, w.L, w.Hkv, n + t - 1, 1, np.array([w.decode_region], np.uint8))
+        O = o.decode_step(1, q, kn[:, :, 0, :][None], vn[:, :, 0, :][None], [w.decode_region])
+        if t == 1 or t == steps:
+            outs.append(O[0])
+    pre_block = list(o.block[0])
+    st, n_ev, ids, logical = o.evict(1, [w.budget_pages[b]])
+    return o, pre_block, st, n_ev[0], logical[0], outs
+
+
+@pytest.mark.parametrize("config,samples", [(4, (0, 15)), (3, (0, 63))])
+def test_full_size_sampled_sequences(config, samples):
+    w = synth.make_workload(config)
+    steps = w.window_k                      # config 3 observes after 16 steps, config 4 after 1
+    g = gpu_run(w, steps)
+    ps = w.page_size
+    for b in samples:
+        o, pre_block, st_o, ne_o, logical_o, outs_o = oracle_run(w, b, steps)
+        assert g["n_ev"][b] == ne_o
+        for og, oo in zip(g["outs"], outs_o):
+            err = float(np.max(np.abs(synth.bf16_to_f64(og[b]) - oo)))
+            assert err <= TOL_O_ABS, (config, b, err)
+        n_pre = g["pre_tokens"][b]
+        P = len(pre_block)
+        assert n_pre == o.n_tokens[0] + ne_o * ps
+        gsl = np.array([g["pre_bt"][b, i // ps] * ps + i % ps for i in range(n_pre)])
+        osl = np.array([pre_block[i // ps] * ps + i % ps for i in range(n_pre)])
+        for key, arr in (("ahat", o.abar), ("a", o.a)):
+            e = rel_err(g[key][gsl], arr[osl])
+            assert e <= TOL_REL, (config, b, key, e)
+        tau = w.tau_scale / n_pre
+        mism = g["t_ref"][gsl] != o.t_ref[osl]
+        assert np.all(np.abs(o.abar[osl][mism] - tau) <= TIE_REL * tau), (config, b, "refresh")
+        e = rel_err(g["prio"][gsl][~mism], o.prio[osl][~mism])
+        assert e <= TOL_REL, (config, b, "prio", e)
+        page_flip = np.zeros(P, bool)
+        page_flip[np.nonzero(mism)[0] // ps] = True
+        S_o = o.page_S[0]
+        e = rel_err(g["page"][b, :P][~page_flip], S_o[~page_flip])
+        assert e <= TOL_REL, (config, b, "page", e)
+        kept = g["bt"][b, :P - ne_o]
+        got = sorted(int(j) for j in np.nonzero(~np.isin(g["pre_bt"][b, :P], kept))[0])
+        assert list(kept) == [g["pre_bt"][b, j] for j in range(P) if j not in set(got)]
+        if got != logical_o:
+            boundary = max(S_o[j] for j in logical_o)
+            for j in set(got) ^ set(logical_o):
+                assert page_flip[j] or abs(S_o[j] - boundary) <= TIE_REL * abs(boundary) + TOL_FLOOR
+        del o
+        gc.collect()

@@ -198,7 +198,7 @@ def test_single_token_and_no_eviction_edges():
     """One cached token (o = v exactly, Abar = 1), and budgets at or above
     the page count (nothing evicted)."""
     w = synth.custom_workload("tiny", L=1, Hq=8, Hkv=2, page_size=16, lengths=[0],
-                              budget_frac=1.0, steps=1, seed=10)
+                              budget_frac=1.0, steps=48, seed=10)
     ls = Lockstep(w)
     ls.decode()
     n = ls.observe(budgets=[5])

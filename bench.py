@@ -368,6 +368,17 @@ def workload_config(w, args):
             "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed}
 
 
+def combine_over_ranks(total_ms: float, tokens_total: float, device):
+    """Whole-job numbers of a replicated run: the timed region is the slowest
+    rank's, the work is the sum over ranks."""
+    import torch
+    t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+    n = torch.tensor([tokens_total], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    torch.distributed.all_reduce(n, op=torch.distributed.ReduceOp.SUM)
+    return float(t.item()), float(n.item())
+
+
 # ------------------------------------------------------------------ main ----
 def main():
     args = parse()
@@ -387,12 +398,7 @@ def main():
     total_ms = r["total_ms"]
     tokens = float(np.mean(r["tokens"]))
     if world > 1:
-        t = torch.tensor([total_ms, tokens * args.steps], dtype=torch.float64, device="cuda")
-        mx = t.clone()
-        torch.distributed.all_reduce(mx[:1], op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.all_reduce(t[1:], op=torch.distributed.ReduceOp.SUM)
-        total_ms = float(mx[0])
-        all_tokens = float(t[1])
+        total_ms, all_tokens = combine_over_ranks(total_ms, tokens * args.steps, "cuda")
     else:
         all_tokens = tokens * args.steps
     if rank != 0:

@@ -235,6 +235,56 @@ md_status md_debug_set(md_ctx *ctx, int key, int64_t value);
 /* Text of the last error on this handle ("" if none). */
 const char *md_last_error(const md_ctx *ctx);
 
+/* ---- stage 1 for callers that cannot allocate device memory ----------- */
+
+/* The paper has no counterpart to this call.  It exists for callers that
+ * cannot call cudaMalloc or any allocating routine: code running where the
+ * allocator is owned by someone else (a serving engine or framework that
+ * hands out only the tensors it allocated), code that must not allocate
+ * between CUDA-graph replays, or embedders whose memory budget is fixed up
+ * front.  Those callers cannot provide md_decode_step's workspace.
+ *
+ * It runs stage 1 alone -- paged GQA decode attention over every cached
+ * token plus each token's attention mass per (layer, KV head) -- over a paged
+ * cache the caller already owns, with md_decode_step's kernel and results.
+ * The kernel's scratch memory (score rows, split partials, arrival counters,
+ * status words) lives in one fixed 24 MiB device array inside the library,
+ * which every GPU that loads the library holds until the process exits.
+ * Nothing is allocated by this call.
+ *
+ *   kv_pool_dev      bf16 [L][num_phys_pages][Hkv][2][page_size][128]: for
+ *                    each (layer, page, KV head) the page's K rows then its V
+ *                    rows (md_decode_step's pool layout; 16-byte aligned)
+ *   block_table_dev  int32 [batch][max_pages_per_seq] physical page ids
+ *   n_tokens_host    [batch] cached tokens per sequence (host), each >= 1 and
+ *                    at most max_pages_per_seq * page_size
+ *   q_dev            bf16 [batch][L][Hq][128]
+ *   out_dev          bf16 [batch][L][Hq][128] (written)
+ *   mass_dev         fp32 [L*Hkv][num_phys_pages*page_size] (written at the
+ *                    slots of cached tokens: sum over the KV head's query heads
+ *                    of their softmax weight on the token)
+ *   stream           cudaStream_t
+ *
+ * Limits: the work must fit the 24 MiB array.  Each (sequence, layer, KV
+ * head) is split into chunks of at most 1,024 tokens, and the partials of all
+ * of them must fit next to the score rows.  Larger work (for instance very
+ * long sequences times many layers and sequences) is rejected with
+ * MD_ERR_CAPACITY before anything is launched; bad arguments with
+ * MD_ERR_INVALID_ARG.
+ *
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress), so make that first call before any stream capture.
+ * Every call on a device shares the same array and clears its counters and
+ * status words on the stream before the kernel; calls whose GPU work overlaps
+ * (other streams, other threads) race on the array and must be serialised by
+ * the caller.  The call is asynchronous and cannot report a device-side wait
+ * timeout; it returns MD_OK once the work is enqueued. */
+md_status md_attend_mass_noalloc(const void *kv_pool_dev, const int32_t *block_table_dev,
+                                 const int32_t *n_tokens_host, const void *q_dev, void *out_dev,
+                                 float *mass_dev, int batch, int num_layers, int num_q_heads,
+                                 int num_kv_heads, int page_size, int max_pages_per_seq,
+                                 int num_phys_pages, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

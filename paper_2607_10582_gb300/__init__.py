@@ -78,6 +78,8 @@ SIGNATURES = {
     "md_profile_read": (_c.c_int, [_P, _P, _P, _c.c_int]),
     "md_debug_set": (_c.c_int, [_P, _c.c_int, _c.c_int64]),
     "md_last_error": (_c.c_char_p, [_P]),
+    "md_attend_mass_noalloc": (_c.c_int, [_P, _P, _P, _P, _P, _P, _c.c_int, _c.c_int, _c.c_int, _c.c_int,
+                                          _c.c_int, _c.c_int, _c.c_int, _P]),
 }
 
 _lib = None

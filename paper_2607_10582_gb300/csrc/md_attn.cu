@@ -552,3 +552,173 @@ cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &tmap, int g
 }
 
 }  // namespace md
+
+/* ------------------------------------------------------------------------ */
+/* Stage 1 without any device allocation.                                   */
+/*                                                                          */
+/* The attention kernel above needs scratch memory besides its inputs and   */
+/* outputs: per-CTA rows of raw scores, the split partials (m, Z, O) of     */
+/* every (sequence, layer, KV head) item and one arrival counter per item.  */
+/* md_decode_step finds them in the caller's workspace.  This variant finds */
+/* them in the fixed array below instead, for callers that cannot allocate  */
+/* device memory at all (see md_attend_mass_noalloc in memdecay.h).         */
+/* ------------------------------------------------------------------------ */
+
+namespace md {
+
+constexpr size_t NOALLOC_BYTES = (size_t)24 << 20;     // 24 MiB, every device that loads us
+constexpr int NOALLOC_TOKENS = 1024;                   // scratch rows per CTA slot
+constexpr size_t NOALLOC_STATUS_BYTES = 256;
+
+static __device__ __align__(256) uint8_t g_noalloc_scratch[NOALLOC_BYTES];
+
+}  // namespace md
+
+#include <math.h>
+#include <string.h>
+
+#include <mutex>
+
+namespace {
+
+/* Device address of g_noalloc_scratch, looked up once per device. */
+std::mutex g_noalloc_mu;
+void *g_noalloc_addr[128] = {nullptr};
+
+cudaError_t noalloc_base(void **out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 128) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_addr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, md::g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_noalloc_addr[dev] = p;
+  }
+  *out = g_noalloc_addr[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" __attribute__((visibility("default"))) md_status md_attend_mass_noalloc(
+    const void *kv_pool_dev, const int32_t *block_table_dev, const int32_t *n_tokens_host,
+    const void *q_dev, void *out_dev, float *mass_dev, int batch, int num_layers,
+    int num_q_heads, int num_kv_heads, int page_size, int max_pages_per_seq, int num_phys_pages,
+    void *stream) {
+  using namespace md;
+  if (!kv_pool_dev || !block_table_dev || !n_tokens_host || !q_dev || !out_dev || !mass_dev)
+    return MD_ERR_INVALID_ARG;
+  if (batch < 1 || batch > MD_MAX_BATCH || num_layers < 1 || num_layers > 255 ||
+      num_kv_heads < 1 || num_q_heads < num_kv_heads || num_q_heads % num_kv_heads ||
+      num_q_heads / num_kv_heads > MD_MAX_GROUP || (page_size != 16 && page_size != 32) ||
+      max_pages_per_seq < 1 || num_phys_pages < 1)
+    return MD_ERR_INVALID_ARG;
+  if ((uintptr_t)kv_pool_dev & 15) return MD_ERR_INVALID_ARG;
+  const long long rows = (long long)num_layers * num_phys_pages * num_kv_heads * 2 * page_size;
+  if (rows >= (1LL << 31)) return MD_ERR_INVALID_ARG;
+  const int ps = page_size;
+  for (int b = 0; b < batch; ++b)
+    if (n_tokens_host[b] < 1 || (long long)n_tokens_host[b] > (long long)max_pages_per_seq * ps)
+      return MD_ERR_INVALID_ARG;
+
+  /* plan: chunks of at most NOALLOC_TOKENS tokens, partials for every chunk
+   * of every item, all inside the fixed array */
+  const long long items = (long long)batch * num_layers * num_kv_heads;
+  int grid_limit = attention_grid_limit(ps);
+  if (grid_limit <= 0) return MD_ERR_CUDA;
+  const size_t scores_bytes = (size_t)grid_limit * 2 * NOALLOC_TOKENS * GP * 4;
+  const size_t counters_bytes = (size_t)((items * 4 + 255) / 256 * 256);
+  if (NOALLOC_STATUS_BYTES + counters_bytes + scores_bytes >= NOALLOC_BYTES) return MD_ERR_CAPACITY;
+  const size_t part_room = NOALLOC_BYTES - NOALLOC_STATUS_BYTES - counters_bytes - scores_bytes;
+  long long cstride = (long long)(part_room / ((size_t)items * PARTIAL_FLOATS * 4));
+  if (cstride > MD_MAX_CHUNKS) cstride = MD_MAX_CHUNKS;
+  const int cap_pages = NOALLOC_TOKENS / ps;
+  AttnParams ap;
+  memset(&ap, 0, sizeof(ap));
+  int Pmax = 1;
+  for (int b = 0; b < batch; ++b) {
+    const int P = (n_tokens_host[b] + ps - 1) / ps;
+    ap.n_pages[b] = P;
+    ap.n_tokens[b] = n_tokens_host[b];
+    if (P > Pmax) Pmax = P;
+  }
+  /* the smallest chunk count that fits the per-chunk cap, then more chunks
+   * while the grid is not yet full and they fit the partials room */
+  int need = (Pmax + cap_pages - 1) / cap_pages;
+  if (need > cstride) return MD_ERR_CAPACITY;
+  int C = need;
+  while (C < cstride && C < Pmax && items * C < grid_limit) ++C;
+  const int T = (Pmax + C - 1) / C;
+  long long U = 0;
+  for (int b = 0; b < batch; ++b) {
+    const int P = ap.n_pages[b];
+    int ch = (P + T - 1) / T;
+    if (ch > C) ch = C;
+    if (ch > P) ch = P;
+    ap.chunks[b] = ch;
+    ap.unit_start[b] = (int)U;
+    U += (long long)num_layers * num_kv_heads * ch;
+  }
+  ap.unit_start[batch] = (int)U;
+  ap.total_units = (int)U;
+  ap.n_seqs = batch;
+
+  void *base = nullptr;
+  cudaError_t e = noalloc_base(&base);
+  if (e != cudaSuccess) return MD_ERR_CUDA;
+  uint8_t *s8 = (uint8_t *)base;
+  ap.status = (int *)s8;
+  ap.counters = (int *)(s8 + NOALLOC_STATUS_BYTES);
+  ap.scratch = (float *)(s8 + NOALLOC_STATUS_BYTES + counters_bytes);
+  ap.partials = (float *)(s8 + NOALLOC_STATUS_BYTES + counters_bytes + scores_bytes);
+  ap.q = (const uint16_t *)q_dev;
+  ap.out = (uint16_t *)out_dev;
+  ap.block_table = block_table_dev;
+  ap.mass = mass_dev;
+  ap.L = num_layers;
+  ap.Hq = num_q_heads;
+  ap.Hkv = num_kv_heads;
+  ap.G = num_q_heads / num_kv_heads;
+  ap.ps = ps;
+  ap.P_phys = num_phys_pages;
+  ap.P_max = max_pages_per_seq;
+  ap.slots = (long long)num_phys_pages * ps;
+  ap.scratch_tokens = NOALLOC_TOKENS;
+  ap.chunk_stride = (int)cstride;
+  ap.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
+  ap.spin_limit_ns = 2000000000LL;
+  ap.extra_arrivals = 0;
+
+  void *fn = nullptr;
+  cudaDriverEntryPointQueryResult qres;
+  e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                       &qres);
+  if (e != cudaSuccess || qres != cudaDriverEntryPointSuccess || !fn) return MD_ERR_CUDA;
+  typedef CUresult (*EncodeFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                               const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                               const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                               CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  CUtensorMap tmap;
+  cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)(2 * ps)};
+  cuuint32_t estr[2] = {1, 1};
+  if (((EncodeFn)fn)(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void *)kv_pool_dev, dims,
+                     strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return MD_ERR_INVALID_ARG;
+
+  /* the array keeps the previous call's contents: counters and status words
+   * must start at zero */
+  cudaStream_t st = (cudaStream_t)stream;
+  e = cudaMemsetAsync(s8, 0, NOALLOC_STATUS_BYTES + counters_bytes, st);
+  if (e != cudaSuccess) return MD_ERR_CUDA;
+  int grid = (int)(U < grid_limit ? U : grid_limit);
+  if (grid < 1) grid = 1;
+  e = launch_attention(ap, tmap, grid, st);
+  return e == cudaSuccess ? MD_OK : MD_ERR_CUDA;
+}

@@ -224,12 +224,24 @@ md_status md_profile_enable(md_ctx *ctx, int enable);
 md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_per_stage,
                           int n_stages);
 
-/* Test support: bounded waits and injected timeouts.
+/* Test and tuning support.
  *   MD_DEBUG_SPIN_LIMIT_NS    limit of each device-side wait (default 2e9)
  *   MD_DEBUG_EXTRA_ARRIVALS   extra arrivals the attention exchange waits for
  *                             on its next launch (a wait nothing completes;
- *                             the kernel then reports MD_ERR_DEVICE_TIMEOUT) */
-enum { MD_DEBUG_SPIN_LIMIT_NS = 0, MD_DEBUG_EXTRA_ARRIVALS = 1 };
+ *                             the kernel then reports MD_ERR_DEVICE_TIMEOUT)
+ *   MD_DEBUG_GRID_LIMIT       cap on the attention kernel's persistent CTAs
+ *                             (0 = all that fit on the device)
+ *   MD_DEBUG_UNIT_OVERHEAD    per-unit cost, in pages, that the attention work
+ *                             planner adds to each chunk (default 8)
+ *   MD_DEBUG_FORCE_CHUNKS     chunks per (sequence, layer, KV head) item
+ *                             (0 = planned; otherwise clamped to the limits) */
+enum {
+  MD_DEBUG_SPIN_LIMIT_NS = 0,
+  MD_DEBUG_EXTRA_ARRIVALS = 1,
+  MD_DEBUG_GRID_LIMIT = 2,
+  MD_DEBUG_UNIT_OVERHEAD = 3,
+  MD_DEBUG_FORCE_CHUNKS = 4
+};
 md_status md_debug_set(md_ctx *ctx, int key, int64_t value);
 
 /* Text of the last error on this handle ("" if none). */

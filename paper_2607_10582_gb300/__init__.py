@@ -39,7 +39,8 @@ MD_HEAD_DIM = 128
  MD_STATE_AHAT, MD_STATE_FREE, MD_STATE_REGION, MD_STATE_WINDOW, MD_STATE_MASS, MD_STATE_POOL) = range(11)
 (MD_QUERY_TOKENS, MD_QUERY_PAGES, MD_QUERY_FREE_TOP, MD_QUERY_STEP, MD_QUERY_WINDOW,
  MD_QUERY_PINNED_PAGES) = range(6)
-MD_DEBUG_SPIN_LIMIT_NS, MD_DEBUG_EXTRA_ARRIVALS = 0, 1
+(MD_DEBUG_SPIN_LIMIT_NS, MD_DEBUG_EXTRA_ARRIVALS, MD_DEBUG_GRID_LIMIT, MD_DEBUG_UNIT_OVERHEAD,
+ MD_DEBUG_FORCE_CHUNKS) = range(5)
 STAGES = ("append", "attention", "fold", "score", "select")
 
 

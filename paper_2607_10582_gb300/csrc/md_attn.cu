@@ -153,12 +153,15 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
 
   if (warp == 0) {
     /* ------------------------------------------------------- producer ---- */
+    /* One thread issues every copy (a single active lane keeps this warp off
+     * the issue slots the consumers need); page ids are loaded eight at a
+     * time so no copy waits on a dependent load. */
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       tma_prefetch_desc(&tmap);
       int i = 0, nu = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x, ++nu) {
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
         const Unit un = decode_unit(p, u);
         /* the unit's G query rows: one bulk copy into a double-buffered slot */
         const int qs = nu & 1;
@@ -170,22 +173,30 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
         bulk_load(sQ_u32 + qs * S::Q_BYTES,
                   p.q + (((size_t)un.b * p.L + un.l) * p.Hq + (size_t)un.kvh * G) * D, G * D * 2,
                   smem_u32(&qfull[qs]));
+        ++nu;
         const int32_t *bt = p.block_table + (size_t)un.b * p.P_max;
-        for (int pg = un.p0; pg < un.p1; ++pg, ++i) {
-          const int s = i % S::R;
-          if (i >= S::R &&
-              !wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
-            ok = false;
-            break;
+        for (int pb = un.p0; pb < un.p1 && ok; pb += 8) {
+          const int cnt = min(8, un.p1 - pb);
+          int ph[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) ph[k] = k < cnt ? bt[pb + k] : 0;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            if (k >= cnt) break;
+            const int s = i % S::R;
+            if (i >= S::R &&
+                !wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
+              ok = false;
+              break;
+            }
+            const int row = (((un.l * p.P_phys + ph[k]) * p.Hkv + un.kvh) * 2) * PS;
+            const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
+            mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
+            tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
+            tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
+            ++i;
           }
-          const int phys = bt[pg];
-          const int row = (((un.l * p.P_phys + phys) * p.Hkv + un.kvh) * 2) * PS;
-          const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
-          mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
-          tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
-          tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
         }
-        if (!ok) { ++nu; break; }
       }
       /* No copy may still be writing this CTA's shared memory when it exits. */
       for (int k = (i > S::R ? i - S::R : 0); k < i; ++k)

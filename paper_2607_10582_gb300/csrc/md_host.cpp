@@ -60,6 +60,9 @@ struct md_ctx {
   std::string err;
   long long spin_limit_ns = 2000000000LL;
   int extra_arrivals = 0;
+  int grid_cap = 0;          // 0: every CTA that fits
+  int unit_overhead = 4;     // planner: per-unit cost in pages
+  int force_chunks = 0;      // planner: 0 = choose
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
   std::vector<ProfRec> pending;
@@ -224,11 +227,22 @@ void plan_attention(const md_ctx *c, int batch, AttnParams &ap, int *grid) {
   for (int b = 0; b < batch; ++b) Pmax = std::max(Pmax, c->n_pages[b]);
   const int max_chunk_pages = std::max(1, c->lay.scratch_tokens / ps);
   const int cmax = c->lay.chunk_stride;
+  const long long glim =
+      c->grid_cap > 0 ? std::min<long long>(c->grid_cap, c->grid_limit) : c->grid_limit;
   double best = 1e300;
   int bestT = 0;
+  /* Every CTA keeps the raw scores of two units in L2 (evict_last) until the
+   * unit after next; keep that set well inside L2 or its lines spill. */
+  const double l2_budget = 56.0 * (1 << 20);
+  for (int pass = 0; pass < 2 && bestT == 0; ++pass)
   for (int C = 1; C <= cmax; ++C) {
     const int T = (Pmax + C - 1) / C;
     if (T > max_chunk_pages) continue;
+    if (pass == 0 && (double)glim * 2 * T * ps * GP * 4 > l2_budget) continue;
+    if (c->force_chunks > 0) {
+      const int need = (Pmax + max_chunk_pages - 1) / max_chunk_pages;
+      if (C != std::min(cmax, std::max(c->force_chunks, need))) continue;
+    }
     long long U = 0;
     int maxpg = 0;
     for (int b = 0; b < batch; ++b) {
@@ -238,14 +252,15 @@ void plan_attention(const md_ctx *c, int batch, AttnParams &ap, int *grid) {
       U += (long long)items * ch;
       maxpg = std::max(maxpg, (P + ch - 1) / ch);
     }
-    const long long G = std::max(1LL, std::min<long long>(U, c->grid_limit));
+    const long long G = std::max(1LL, std::min<long long>(U, glim));
     const double rounds = (double)((U + G - 1) / G);
-    const double cost = rounds * (maxpg + 2.0);
+    const double cost = rounds * (maxpg + (double)c->unit_overhead);
     if (cost < best - 1e-9) {
       best = cost;
       bestT = T;
     }
   }
+  if (bestT == 0) bestT = max_chunk_pages;
   long long U = 0;
   for (int b = 0; b < batch; ++b) {
     const int P = c->n_pages[b];
@@ -260,7 +275,7 @@ void plan_attention(const md_ctx *c, int batch, AttnParams &ap, int *grid) {
   ap.unit_start[batch] = (int)U;
   ap.total_units = (int)U;
   ap.n_seqs = batch;
-  *grid = (int)std::max(1LL, std::min<long long>(U, c->grid_limit));
+  *grid = (int)std::max(1LL, std::min<long long>(U, glim));
 }
 
 bool valid_region(int r) { return r >= 0 && r < MD_NUM_REGIONS; }
@@ -903,6 +918,21 @@ MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
   if (key == MD_DEBUG_EXTRA_ARRIVALS) {
     if (value < 0 || value > 1000) return fail(c, MD_ERR_INVALID_ARG, "extra arrivals out of range");
     c->extra_arrivals = (int)value;
+    return MD_OK;
+  }
+  if (key == MD_DEBUG_GRID_LIMIT) {
+    if (value < 0) return fail(c, MD_ERR_INVALID_ARG, "negative grid limit");
+    c->grid_cap = (int)std::min<int64_t>(value, MAX_GRID);
+    return MD_OK;
+  }
+  if (key == MD_DEBUG_UNIT_OVERHEAD) {
+    if (value < 0 || value > 4096) return fail(c, MD_ERR_INVALID_ARG, "unit overhead out of range");
+    c->unit_overhead = (int)value;
+    return MD_OK;
+  }
+  if (key == MD_DEBUG_FORCE_CHUNKS) {
+    if (value < 0 || value > MD_MAX_CHUNKS) return fail(c, MD_ERR_INVALID_ARG, "chunk count out of range");
+    c->force_chunks = (int)value;
     return MD_OK;
   }
   return fail(c, MD_ERR_INVALID_ARG, "unknown debug key");

@@ -15,7 +15,7 @@ namespace md {
 constexpr int D = MD_HEAD_DIM;
 constexpr int GP = MD_MAX_GROUP;            // query heads per KV head, padded
 constexpr int PARTIAL_FLOATS = 1088;        // m[8] l[8] O[8][128], padded to 256 B
-constexpr int MAX_GRID = 256;               // persistent attention CTAs (>= SM count)
+constexpr int MAX_GRID = 512;               // persistent attention CTAs (>= 2 x SM count)
 
 enum DevStatus { ST_CODE = 0, ST_ABORT = 1, ST_DIAG = 2, ST_WORDS = 8 };
 

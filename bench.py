@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--max-tokens", type=int, default=0,
                     help="truncate every trace to this many tokens (small profiling cases)")
+    ap.add_argument("--layerwise", action="store_true",
+                    help="decode through md_decode_layer, one call per layer")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -197,8 +199,25 @@ def run_native(args, rank, world, local_rank):
     torch.cuda.synchronize()
     budgets = list(w.budget_pages)
 
+    # tensors a step reads from the host in the end-to-end measurement
+    step_inputs = [q, kn, vn]
+    step_output = out
+    if args.layerwise:
+        # a model hands each layer its own contiguous [B][heads][D] tensors
+        q_lm = q.permute(1, 0, 2, 3).contiguous()
+        kn_lm = kn.permute(1, 0, 2, 3).contiguous()
+        vn_lm = vn.permute(1, 0, 2, 3).contiguous()
+        out_lm = torch.empty((L, B, Hq, D), dtype=torch.int16, device=dev)
+        q_l, kn_l, vn_l, out_l = list(q_lm), list(kn_lm), list(vn_lm), list(out_lm)
+        step_inputs = [q_lm, kn_lm, vn_lm]
+        step_output = out_lm
+
     def one_step():
-        cache.decode_step(B, q, kn, vn, regs, out)
+        if args.layerwise:
+            for l in range(L):
+                cache.decode_layer(l, B, q_l[l], kn_l[l], vn_l[l], regs, out_l[l])
+        else:
+            cache.decode_step(B, q, kn, vn, regs, out)
         # observation every window_k steps (k = 1 for configs 0-2 and 4)
         if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
             cache.evict(budgets)
@@ -255,25 +274,22 @@ def run_native(args, rank, world, local_rank):
     # ---- end to end through the C ABI with host buffers ----
     e2e = None
     if not args.no_e2e:
-        qh = q.cpu().pin_memory()
-        knh = kn.cpu().pin_memory()
-        vnh = vn.cpu().pin_memory()
-        outh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+        hosts = [t.cpu().pin_memory() for t in step_inputs]
+        outh = torch.empty(step_output.shape, dtype=step_output.dtype).pin_memory()
         e_ms = []
         for i in range(args.warmup + args.steps):
             if restore:
                 cache.load_state(saved)
             torch.cuda.synchronize()
             t0 = time.perf_counter()
-            q.copy_(qh, non_blocking=True)
-            kn.copy_(knh, non_blocking=True)
-            vn.copy_(vnh, non_blocking=True)
+            for d_t, h_t in zip(step_inputs, hosts):
+                d_t.copy_(h_t, non_blocking=True)
             one_step()
-            outh.copy_(out, non_blocking=True)
+            outh.copy_(step_output, non_blocking=True)
             torch.cuda.synchronize()
             if i >= args.warmup:
                 e_ms.append((time.perf_counter() - t0) * 1e3)
-        h2d = (qh.numel() + knh.numel() + vnh.numel()) * 2 + B
+        h2d = sum(h_t.numel() for h_t in hosts) * 2 + B
         d2h = outh.numel() * 2
         e2e = {"ms_per_step": float(np.mean(e_ms)), "tokens_per_step": tok_per_step[0],
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
@@ -365,7 +381,8 @@ def workload_config(w, args):
             "phase": "full-trace step (state restored before each step)" if args.phase == "full"
             else "steady state",
             "l2": "no flush: inputs larger than L2 (K/V read per step >> 129 MB)",
-            "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed}
+            "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed,
+            "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict"}
 
 
 def combine_over_ranks(total_ms: float, tokens_total: float, device):
@@ -412,17 +429,20 @@ def main():
     kv_bytes = tokens * r["kv_bytes_per_token"]
     qo_bytes = 2 * w.B * w.L * w.Hq * w.D * 2
     attn_bytes = kv_bytes + qo_bytes
+    launches_per_step = max(1, r["attn_n"] // args.steps)     # L with --layerwise, else 1
     attn_avg_s = r["attn_ms"] / max(1, r["attn_n"]) / 1e3
-    achieved = attn_bytes / attn_avg_s / 1e9
+    bytes_per_launch = attn_bytes / launches_per_step
+    achieved = bytes_per_launch / attn_avg_s / 1e9
     tpt = ncu_traffic_per_token()
-    traffic = None if tpt is None else tpt * tokens * w.L
+    traffic = None if tpt is None else tpt * tokens * w.L / launches_per_step
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload_config(w, args),
         "roofline": {"bound": "hbm", "kernel": "attn_mass_kernel (stage 1)", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{peak_kind} copy",
-                     "traffic": traffic, "algorithmic_bytes": attn_bytes,
+                     "traffic": traffic, "algorithmic_bytes": bytes_per_launch,
+                     "launches_per_step": launches_per_step,
                      "frac_of_8TBps_spec": achieved / SPEC_HBM_GBS},
         "step_hbm_fraction": {"algorithmic_GBps": attn_bytes / (ms_per_step / 1e3) / 1e9,
                               "frac_measured": attn_bytes / (ms_per_step / 1e3) / 1e9 / peak,

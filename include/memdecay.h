@@ -145,6 +145,24 @@ md_status md_append_tokens(md_ctx *ctx, int seq, int n_tokens, const uint8_t *re
 md_status md_decode_step(md_ctx *ctx, int batch, const void *q_dev, const void *k_new_dev,
                          const void *v_new_dev, const uint8_t *new_region_host, void *out_dev);
 
+/* The same decode step, one layer per call, for a model that runs its other
+ * per-layer work (MLP, norms) between the layers' attentions: the production
+ * shape of the loop (Fig. 1: the decode engine appends KV and attends layer
+ * by layer; Sec. III-C: the mass is gathered over all layers).  Call it for
+ * layers 0, 1, ..., L-1 in order; after the call for layer L-1 the step is
+ * complete and equivalent to md_decode_step.  Layer 0 advances the step
+ * counter, takes new pages and starts the new tokens' state (it reads
+ * new_region_host); every layer writes its own K/V row of the new tokens and
+ * runs stage 1 for that layer only.  While a step is in progress, calls other
+ * than the next layer return MD_ERR_STATE.
+ *   q_dev                bf16 [batch][Hq][D]   (this layer)
+ *   k_new_dev, v_new_dev bf16 [batch][Hkv][D]  (this layer)
+ *   new_region_host      [batch]               (host; read at layer 0)
+ *   out_dev              bf16 [batch][Hq][D]   (written) */
+md_status md_decode_layer(md_ctx *ctx, int layer, int batch, const void *q_dev,
+                          const void *k_new_dev, const void *v_new_dev,
+                          const uint8_t *new_region_host, void *out_dev);
+
 /* The observation step of Algorithm 1 for sequences [0, batch): stages 2-4.
  * If decode steps ran since the last call, Abar_i = (attention mass summed
  * over those k steps, layers and query heads) / (k L Hq), then Eq. 2, Eq. 3

@@ -66,6 +66,7 @@ SIGNATURES = {
     "md_set_region_params": (_c.c_int, [_P, _c.c_int, _c.c_float, _c.c_float, _c.c_int]),
     "md_append_tokens": (_c.c_int, [_P, _c.c_int, _c.c_int, _P, _P, _P, _P]),
     "md_decode_step": (_c.c_int, [_P, _c.c_int, _P, _P, _P, _P, _P]),
+    "md_decode_layer": (_c.c_int, [_P, _c.c_int, _c.c_int, _P, _P, _P, _P, _P]),
     "md_evict": (_c.c_int, [_P, _c.c_int, _P, _P, _P]),
     "md_sync": (_c.c_int, [_P]),
     "md_destroy": (_c.c_int, [_P]),
@@ -194,6 +195,11 @@ class Cache:
     def decode_step(self, batch: int, q, k_new, v_new, new_regions, out):
         regs, rp = _host(new_regions, np.uint8)
         return self._check(lib().md_decode_step(self.h, batch, _ptr(q), _ptr(k_new), _ptr(v_new), rp, _ptr(out)))
+
+    def decode_layer(self, layer: int, batch: int, q, k_new, v_new, new_regions, out):
+        regs, rp = _host(new_regions, np.uint8)
+        return self._check(lib().md_decode_layer(self.h, layer, batch, _ptr(q), _ptr(k_new), _ptr(v_new), rp,
+                                                 _ptr(out)))
 
     def evict(self, budgets: Sequence[int], evicted_ids=None):
         bud, bp = _host(budgets, np.int32)

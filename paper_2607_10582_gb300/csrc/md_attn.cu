@@ -68,8 +68,9 @@ __device__ __forceinline__ Unit decode_unit(const AttnParams &p, int u) {
   int rem = u - p.unit_start[lo];
   int item = rem / un.C;
   un.j = rem - item * un.C;
-  un.l = item / p.Hkv;
-  un.kvh = item - un.l * p.Hkv;
+  const int ll = item / p.Hkv;
+  un.kvh = item - ll * p.Hkv;
+  un.l = p.l0 + ll;
   int P = p.n_pages[lo];
   un.p0 = (int)(((long long)un.j * P) / un.C);
   un.p1 = (int)(((long long)(un.j + 1) * P) / un.C);
@@ -171,7 +172,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
         }
         mbar_arrive_expect_tx(smem_u32(&qfull[qs]), G * D * 2);
         bulk_load(sQ_u32 + qs * S::Q_BYTES,
-                  p.q + (((size_t)un.b * p.L + un.l) * p.Hq + (size_t)un.kvh * G) * D, G * D * 2,
+                  p.q + (((size_t)un.b * p.q_layers + (un.l - p.l0)) * p.Hq + (size_t)un.kvh * G) * D, G * D * 2,
                   smem_u32(&qfull[qs]));
         ++nu;
         const int32_t *bt = p.block_table + (size_t)un.b * p.P_max;
@@ -281,7 +282,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       const int E = G * D;
       const int lo = (int)(((long long)pv.j * E) / C);
       const int hi = (int)(((long long)(pv.j + 1) * E) / C);
-      uint16_t *orow = p.out + (((size_t)pv.b * p.L + pv.l) * p.Hq + (size_t)pv.kvh * G) * D;
+      uint16_t *orow = p.out + (((size_t)pv.b * p.q_layers + (pv.l - p.l0)) * p.Hq + (size_t)pv.kvh * G) * D;
       const int q4 = ct & 3;
       for (int e0 = lo; e0 < hi; e0 += NC / 4) {
         const int e = e0 + (ct >> 2);
@@ -690,6 +691,9 @@ extern "C" __attribute__((visibility("default"))) md_status md_attend_mass_noall
   ap.block_table = block_table_dev;
   ap.mass = mass_dev;
   ap.L = num_layers;
+  ap.l0 = 0;
+  ap.L_launch = num_layers;
+  ap.q_layers = num_layers;
   ap.Hq = num_q_heads;
   ap.Hkv = num_kv_heads;
   ap.G = num_q_heads / num_kv_heads;

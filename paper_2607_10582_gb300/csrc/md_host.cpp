@@ -40,6 +40,8 @@ struct HostMirror {
   int window_steps = 0, window_batch = 0;
   int mass_pending = 0, mass_batch = 0;
   int64_t free_top = 0;
+  int layer_next = 0;     // md_decode_layer: next layer expected (0 = none in progress)
+  int layer_batch = 0;
 };
 
 }  // namespace
@@ -220,9 +222,9 @@ md_status launch_fold(md_ctx *c) {
 /* Split every (sequence, layer, KV head) item's pages into chunks so that the
  * persistent grid gets balanced rounds: minimise rounds x (largest chunk +
  * a per-unit overhead), with at most MD_MAX_CHUNK_TOKENS tokens per chunk. */
-void plan_attention(const md_ctx *c, int batch, AttnParams &ap, int *grid) {
+void plan_attention(const md_ctx *c, int batch, int layers, AttnParams &ap, int *grid) {
   const int ps = c->cfg.page_size;
-  const int items = c->cfg.num_layers * c->cfg.num_kv_heads;
+  const int items = layers * c->cfg.num_kv_heads;
   int Pmax = 1;
   for (int b = 0; b < batch; ++b) Pmax = std::max(Pmax, c->n_pages[b]);
   const int max_chunk_pages = std::max(1, c->lay.scratch_tokens / ps);
@@ -425,6 +427,7 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
                                   const void *v_dev) {
   if (!c) return MD_ERR_INVALID_ARG;
   if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  if (c->m.layer_next != 0) return fail(c, MD_ERR_STATE, "a layer-by-layer step is in progress");
   const md_config &cf = c->cfg;
   if (seq < 0 || seq >= cf.max_batch) return fail(c, MD_ERR_INVALID_ARG, "seq out of range");
   if (n < 0) return fail(c, MD_ERR_INVALID_ARG, "negative token count");
@@ -479,6 +482,9 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
   ap.ps = ps;
   ap.P_phys = cf.num_phys_pages;
   ap.P_max = cf.max_pages_per_seq;
+  ap.l0 = 0;
+  ap.init_state = 1;
+  ap.lookup_only = 0;
   ap.n_seqs = 1;
   ap.n_per_seq = n;
   ap.seq0 = seq;
@@ -495,15 +501,13 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
   return MD_OK;
 }
 
-MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const void *k_new,
-                                const void *v_new, const uint8_t *new_region_host,
-                                void *out_dev) {
-  if (!c) return MD_ERR_INVALID_ARG;
-  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+namespace {
+
+/* Checks shared by md_decode_step and layer 0 of md_decode_layer. */
+md_status check_step(md_ctx *c, int batch, const uint8_t *new_region_host) {
   const md_config &cf = c->cfg;
   if (batch < 1 || batch > cf.max_batch) return fail(c, MD_ERR_INVALID_ARG, "batch out of range");
-  if (!q_dev || !k_new || !v_new || !new_region_host || !out_dev)
-    return fail(c, MD_ERR_INVALID_ARG, "null pointer");
+  if (!new_region_host) return fail(c, MD_ERR_INVALID_ARG, "null pointer");
   if (c->m.window_steps > 0 && batch != c->m.window_batch)
     return fail(c, MD_ERR_INVALID_ARG, "batch changed inside an observation window");
   const int ps = cf.page_size;
@@ -517,14 +521,11 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   }
   if (need_total > c->m.free_top) return fail(c, MD_ERR_CAPACITY, "page pool exhausted");
   if (c->m.t + 1 >= (1LL << 31)) return fail(c, MD_ERR_STATE, "step counter overflow");
+  return MD_OK;
+}
 
-  if (c->m.mass_pending) {
-    md_status st = launch_fold(c);
-    if (st != MD_OK) return st;
-  }
-  c->m.t += 1;
-  /* stage 0: append the new tokens */
-  AppendParams ap;
+void fill_append_common(md_ctx *c, AppendParams &ap) {
+  const md_config &cf = c->cfg;
   memset(&ap, 0, sizeof(ap));
   ap.pool = ptr<uint16_t>(c, c->lay.pool);
   ap.block_table = ptr<int32_t>(c, c->lay.block_table);
@@ -535,20 +536,37 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   ap.ahat = ptr<float>(c, c->lay.ahat);
   ap.prio = ptr<float>(c, c->lay.prio);
   ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
-  ap.k_src = (const uint16_t *)k_new;
-  ap.v_src = (const uint16_t *)v_new;
-  ap.sb = (long long)cf.num_layers * cf.num_kv_heads * D;
-  ap.sl = (long long)cf.num_kv_heads * D;
-  ap.sh = D;
-  ap.si = 0;
-  ap.L = cf.num_layers;
   ap.Hkv = cf.num_kv_heads;
-  ap.ps = ps;
+  ap.ps = cf.page_size;
   ap.P_phys = cf.num_phys_pages;
   ap.P_max = cf.max_pages_per_seq;
-  ap.n_seqs = batch;
   ap.n_per_seq = 1;
   ap.seq0 = 0;
+}
+
+/* Start of a decode step: advance t, take the new pages, append the new
+ * tokens' K/V for layers [l0, l0 + L) and start their state. */
+md_status begin_step(md_ctx *c, int batch, int l0, int L, long long sb, long long sl,
+                     const void *k_new, const void *v_new, const uint8_t *new_region_host) {
+  const int ps = c->cfg.page_size;
+  if (c->m.mass_pending) {
+    md_status st = launch_fold(c);
+    if (st != MD_OK) return st;
+  }
+  c->m.t += 1;
+  AppendParams ap;
+  fill_append_common(c, ap);
+  ap.k_src = (const uint16_t *)k_new;
+  ap.v_src = (const uint16_t *)v_new;
+  ap.sb = sb;
+  ap.sl = sl;
+  ap.sh = D;
+  ap.si = 0;
+  ap.L = L;
+  ap.l0 = l0;
+  ap.init_state = 1;
+  ap.lookup_only = 0;
+  ap.n_seqs = batch;
   ap.insert_step = (int)c->m.t;
   long long popped = 0;
   for (int b = 0; b < batch; ++b) {
@@ -564,8 +582,13 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   if (e != cudaSuccess) return cuda_fail(c, e, "append launch");
   for (int b = 0; b < batch; ++b) mirror_token(c, b, new_region_host[b]);
   c->m.free_top -= popped;
+  return MD_OK;
+}
 
-  /* stage 1: attention + mass */
+/* Stage 1 over layers [l0, l0 + L); q/out hold q_layers layers. */
+md_status run_attention(md_ctx *c, int batch, int l0, int L, int q_layers, const void *q_dev,
+                        void *out_dev) {
+  const md_config &cf = c->cfg;
   AttnParams atp;
   memset(&atp, 0, sizeof(atp));
   atp.q = (const uint16_t *)q_dev;
@@ -577,10 +600,13 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   atp.counters = ptr<int>(c, c->lay.counters);
   atp.status = ptr<int>(c, c->lay.status);
   atp.L = cf.num_layers;
+  atp.l0 = l0;
+  atp.L_launch = L;
+  atp.q_layers = q_layers;
   atp.Hq = cf.num_q_heads;
   atp.Hkv = cf.num_kv_heads;
   atp.G = cf.num_q_heads / cf.num_kv_heads;
-  atp.ps = ps;
+  atp.ps = cf.page_size;
   atp.P_phys = cf.num_phys_pages;
   atp.P_max = cf.max_pages_per_seq;
   atp.slots = (long long)c->lay.slots;
@@ -591,15 +617,91 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   atp.extra_arrivals = c->extra_arrivals;
   c->extra_arrivals = 0;
   int grid = 1;
-  plan_attention(c, batch, atp, &grid);
+  plan_attention(c, batch, L, atp, &grid);
+  cudaEvent_t e0;
   prof_begin(c, &e0);
-  e = launch_attention(atp, c->tmap, grid, c->stream);
+  cudaError_t e = launch_attention(atp, c->tmap, grid, c->stream);
   prof_end(c, STAGE_ATTN, e0);
   if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
+  return MD_OK;
+}
+
+void end_step(md_ctx *c, int batch) {
   c->m.mass_pending = 1;
   c->m.mass_batch = batch;
   c->m.window_steps += 1;
   c->m.window_batch = batch;
+}
+
+}  // namespace
+
+MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const void *k_new,
+                                const void *v_new, const uint8_t *new_region_host,
+                                void *out_dev) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  if (c->m.layer_next != 0) return fail(c, MD_ERR_STATE, "a layer-by-layer step is in progress");
+  if (!q_dev || !k_new || !v_new || !out_dev) return fail(c, MD_ERR_INVALID_ARG, "null pointer");
+  md_status st = check_step(c, batch, new_region_host);
+  if (st != MD_OK) return st;
+  const md_config &cf = c->cfg;
+  st = begin_step(c, batch, 0, cf.num_layers, (long long)cf.num_layers * cf.num_kv_heads * D,
+                  (long long)cf.num_kv_heads * D, k_new, v_new, new_region_host);
+  if (st != MD_OK) return st;
+  st = run_attention(c, batch, 0, cf.num_layers, cf.num_layers, q_dev, out_dev);
+  if (st != MD_OK) return st;
+  end_step(c, batch);
+  return MD_OK;
+}
+
+MD_API md_status md_decode_layer(md_ctx *c, int layer, int batch, const void *q_dev,
+                                 const void *k_new, const void *v_new,
+                                 const uint8_t *new_region_host, void *out_dev) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  const md_config &cf = c->cfg;
+  if (!q_dev || !k_new || !v_new || !out_dev) return fail(c, MD_ERR_INVALID_ARG, "null pointer");
+  if (layer != c->m.layer_next)
+    return fail(c, MD_ERR_STATE, "layer %d called, layer %d expected", layer, c->m.layer_next);
+  md_status st;
+  if (layer == 0) {
+    st = check_step(c, batch, new_region_host);
+    if (st != MD_OK) return st;
+    st = begin_step(c, batch, 0, 1, (long long)cf.num_kv_heads * D, 0, k_new, v_new,
+                    new_region_host);
+    if (st != MD_OK) return st;
+    c->m.layer_batch = batch;
+  } else {
+    if (batch != c->m.layer_batch)
+      return fail(c, MD_ERR_INVALID_ARG, "batch changed within a decode step");
+    /* the new tokens' pages and state exist: write this layer's K/V only */
+    AppendParams ap;
+    fill_append_common(c, ap);
+    ap.k_src = (const uint16_t *)k_new;
+    ap.v_src = (const uint16_t *)v_new;
+    ap.sb = (long long)cf.num_kv_heads * D;
+    ap.sl = 0;
+    ap.sh = D;
+    ap.si = 0;
+    ap.L = 1;
+    ap.l0 = layer;
+    ap.init_state = 0;
+    ap.lookup_only = 1;
+    ap.n_seqs = batch;
+    for (int b = 0; b < batch; ++b) ap.tok0[b] = (int)c->n_tokens[b] - 1;
+    cudaEvent_t e0;
+    prof_begin(c, &e0);
+    cudaError_t e = launch_append(ap, c->stream);
+    prof_end(c, STAGE_APPEND, e0);
+    if (e != cudaSuccess) return cuda_fail(c, e, "append launch");
+  }
+  st = run_attention(c, batch, layer, 1, 1, q_dev, out_dev);
+  if (st != MD_OK) return st;
+  c->m.layer_next = layer + 1;
+  if (c->m.layer_next == cf.num_layers) {
+    c->m.layer_next = 0;
+    end_step(c, batch);
+  }
   return MD_OK;
 }
 
@@ -607,6 +709,7 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
                           int32_t *evicted_ids_dev) {
   if (!c) return MD_ERR_INVALID_ARG;
   if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  if (c->m.layer_next != 0) return fail(c, MD_ERR_STATE, "a layer-by-layer step is in progress");
   const md_config &cf = c->cfg;
   if (batch < 1 || batch > cf.max_batch) return fail(c, MD_ERR_INVALID_ARG, "batch out of range");
   if (!budget) return fail(c, MD_ERR_INVALID_ARG, "null budget");
@@ -822,7 +925,7 @@ MD_API md_status md_state_bytes(const md_ctx *c, size_t *dev_bytes, size_t *host
 
 MD_API md_status md_save_state(md_ctx *c, void *dst_dev, void *host_blob) {
   if (!c || !dst_dev || !host_blob) return MD_ERR_INVALID_ARG;
-  if (c->m.window_steps != 0 || c->m.mass_pending)
+  if (c->m.window_steps != 0 || c->m.mass_pending || c->m.layer_next != 0)
     return fail(c, MD_ERR_STATE, "checkpoint only between observation windows");
   size_t pos = 0, off, n;
   for (int w : SAVED) {

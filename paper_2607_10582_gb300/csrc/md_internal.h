@@ -47,7 +47,10 @@ struct AppendParams {
   long long sb, sl, sh, si;              // element strides of the source (seq, layer, head, token)
   const uint8_t *regions_dev;            // per token (prefill) or null
   const int32_t *steps_dev;              // per token (prefill) or null
-  int L, Hkv, ps, P_phys, P_max;
+  int L, Hkv, ps, P_phys, P_max;         // L: layers written by this launch
+  int l0;                                // first pool layer written
+  int init_state;                        // 1: start token state, record new pages
+  int lookup_only;                       // 1: pages already in the block table
   int n_seqs, n_per_seq, seq0, insert_step;
   int tok0[MD_MAX_BATCH];                // cached tokens before this append
   int pop_base[MD_MAX_BATCH];            // free-stack index of the first page taken
@@ -65,7 +68,9 @@ struct AttnParams {
   float *partials;     // [items][chunk_stride][PARTIAL_FLOATS]
   int *counters;       // [items]
   int *status;         // sticky device status words
-  int L, Hq, Hkv, G, ps, P_phys, P_max;
+  int L, Hq, Hkv, G, ps, P_phys, P_max;   // L: layers of the model
+  int l0, L_launch;    // layers [l0, l0 + L_launch) attended by this launch
+  int q_layers;        // layers held by the q / out tensors (L or 1)
   long long slots;
   int scratch_tokens;  // scratch row capacity per CTA slot (tokens)
   int chunk_stride;    // partial slots reserved per item

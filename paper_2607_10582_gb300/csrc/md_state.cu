@@ -60,7 +60,7 @@ __global__ void append_kernel(const __grid_constant__ AppendParams p) {
     const int seq = p.seq0 + j;
     const int tok = p.tok0[j] + i;
     const int pg = tok / p.ps, off = tok - pg * p.ps;
-    const int pages_before = (p.tok0[j] + p.ps - 1) / p.ps;
+    const int pages_before = p.lookup_only ? 0x7fffffff : (p.tok0[j] + p.ps - 1) / p.ps;
     int phys;
     if (pg < pages_before)
       phys = p.block_table[(size_t)seq * p.P_max + pg];
@@ -70,11 +70,11 @@ __global__ void append_kernel(const __grid_constant__ AppendParams p) {
     const uint16_t *src = (kv == 0 ? p.k_src : p.v_src) + (long long)j * p.sb +
                           (long long)l * p.sl + (long long)h * p.sh + (long long)i * p.si;
     uint16_t *dst = p.pool +
-                    ((((size_t)l * p.P_phys + phys) * p.Hkv + h) * 2 + kv) * (size_t)p.ps * D +
+                    ((((size_t)(p.l0 + l) * p.P_phys + phys) * p.Hkv + h) * 2 + kv) * (size_t)p.ps * D +
                     (size_t)off * D;
     ((uint4 *)dst)[c] = ((const uint4 *)src)[c];
 
-    if (c == 0 && kv == 0 && h == 0 && l == 0) {
+    if (p.init_state && c == 0 && kv == 0 && h == 0 && l == 0) {
       const size_t slot = (size_t)phys * p.ps + off;
       p.region[slot] = p.regions_dev ? p.regions_dev[i] : p.regions_param[j];
       p.t_ref[slot] = p.steps_dev ? p.steps_dev[i] : p.insert_step;
@@ -106,6 +106,23 @@ __device__ __forceinline__ int find_seq(const int *start, int n, int x) {
   return lo;
 }
 
+/* Sum of one token's mass over the rows (layer, KV head) in a fixed order,
+ * four partial sums so that many row loads are in flight per lane. */
+__device__ __forceinline__ float sum_rows(const float *mass, long long slots, int rows, size_t slot) {
+  float w0 = 0.f, w1 = 0.f, w2 = 0.f, w3 = 0.f;
+  const float *m = mass + slot;
+  int r = 0;
+#pragma unroll 4
+  for (; r + 4 <= rows; r += 4) {
+    w0 += __ldcs(m + (size_t)r * slots);
+    w1 += __ldcs(m + (size_t)(r + 1) * slots);
+    w2 += __ldcs(m + (size_t)(r + 2) * slots);
+    w3 += __ldcs(m + (size_t)(r + 3) * slots);
+  }
+  for (; r < rows; ++r) w0 += __ldcs(m + (size_t)r * slots);
+  return (w0 + w1) + (w2 + w3);
+}
+
 /* Each warp handles 32/PS consecutive pages per iteration, one lane per
  * token slot; the loop count is uniform across the warp so the segmented
  * shuffle reductions see every lane. */
@@ -134,17 +151,14 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
     int pinned = 0;
     if (valid) {
       if (p.fold_only) {
-        float w = p.window[slot];
-        for (int r = 0; r < p.rows; ++r) w += p.mass[(size_t)r * p.slots + slot];
-        p.window[slot] = w;
+        p.window[slot] += sum_rows(p.mass, p.slots, p.rows, slot);
       } else {
         const int reg = p.region[slot];
         float a = p.a[slot];
         int tr = p.t_ref[slot];
         if (p.observe) {
           float w = p.window[slot];
-          if (p.mass_pending)
-            for (int r = 0; r < p.rows; ++r) w += p.mass[(size_t)r * p.slots + slot];
+          if (p.mass_pending) w += sum_rows(p.mass, p.slots, p.rows, slot);
           const float abar = __fdiv_rn(w, p.norm);                    // Sec. III-C
           a = p.rho * a + p.gamma * abar;                             // Eq. 2
           const float tau = __fdiv_rn(p.tau_scale, (float)p.n_tokens[b]);

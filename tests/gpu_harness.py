@@ -48,8 +48,9 @@ def rel_err(g, o):
 
 
 class Lockstep:
-    def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2):
+    def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2, layerwise=False):
         self.w = w
+        self.layerwise = layerwise
         B = w.B
         self.P_max = w.max_pages_per_seq()
         self.P_phys = w.num_phys_pages() + phys_slack
@@ -85,7 +86,15 @@ class Lockstep:
         q = synth.q_host(w.seed, B, w.L, w.Hq, w.Hkv, t, w.structured)
         kn, vn = synth.step_kv_host(w.seed, self.pos, regions, w.L, w.Hkv, w.structured)
         out = torch.empty((B, w.L, w.Hq, w.D), dtype=torch.int16, device="cuda")
-        self.gpu.decode_step(B, to_dev(q), to_dev(kn), to_dev(vn), regions, out)
+        if self.layerwise:
+            qd, knd, vnd = to_dev(q), to_dev(kn), to_dev(vn)
+            for l in range(w.L):
+                o_l = torch.empty((B, w.Hq, w.D), dtype=torch.int16, device="cuda")
+                self.gpu.decode_layer(l, B, qd[:, l].contiguous(), knd[:, l].contiguous(),
+                                      vnd[:, l].contiguous(), regions, o_l)
+                out[:, l] = o_l
+        else:
+            self.gpu.decode_step(B, to_dev(q), to_dev(kn), to_dev(vn), regions, out)
         O = self.orc.decode_step(B, q, kn, vn, regions)
         for b in range(B):
             self.pos[b] += 1

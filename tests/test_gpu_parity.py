@@ -99,6 +99,36 @@ def test_pins_over_budget_warns():
     assert st == md.MD_WARN_OVER_BUDGET
 
 
+def test_layer_by_layer_decode():
+    """md_decode_layer, one layer per call (the shape a real model with MLPs
+    between layers uses), matches the oracle's whole decode step."""
+    w = synth.custom_workload("layers", L=3, Hq=16, Hkv=2, page_size=16, lengths=[500, 2200],
+                              budget_frac=0.4, steps=10, seed=12, structured=True)
+    ls = Lockstep(w, layerwise=True).run()
+    ls.check_layout()
+    w4 = synth.custom_workload("layers4", L=4, Hq=12, Hkv=2, page_size=32, lengths=[1300],
+                               budget_frac=0.5, steps=6, seed=13, window_k=3)
+    Lockstep(w4, layerwise=True).run().check_layout()
+
+
+def test_layer_by_layer_call_order_is_enforced():
+    c = md.Cache(2, 8, 2, 16, 1, 8, 16)
+    z = torch.zeros((1, 8, 128), dtype=torch.int16, device="cuda")
+    zk = torch.zeros((1, 2, 128), dtype=torch.int16, device="cuda")
+    with pytest.raises(md.MemDecayError) as e:
+        c.decode_layer(1, 1, z, zk, zk, [6], z)
+    assert e.value.status == md.MD_ERR_STATE
+    c.decode_layer(0, 1, z, zk, zk, [6], z)
+    for call in (lambda: c.evict([4]), lambda: c.decode_layer(0, 1, z, zk, zk, [6], z)):
+        with pytest.raises(md.MemDecayError) as e:
+            call()
+        assert e.value.status == md.MD_ERR_STATE
+    c.decode_layer(1, 1, z, zk, zk, [6], z)
+    st, n = c.evict([4])
+    assert st == md.MD_OK and c.query(md.MD_QUERY_TOKENS, 0) == 1
+    assert c.sync() == md.MD_OK
+
+
 def test_config1_first_steps():
     """Config 1 geometry (Qwen2.5-1.5B, 28 layers, 12/2 heads), 1,700 tokens."""
     ls = Lockstep(synth.make_workload(1))

@@ -127,6 +127,56 @@ def select_pages_min_heap(S32: Sequence[float], evictable: Sequence[bool], n_evi
     return sorted(out)
 
 
+CALIB_BUCKET_WIDTH = 4      # Fig. 3: age buckets of 4 decode steps
+CALIB_BUCKETS = 256         # ages 0 .. 1023 steps
+
+
+def age_bucket(age: int, width: int = CALIB_BUCKET_WIDTH) -> int:
+    """Age bucket of a token of age `age` (decode steps since insertion)."""
+    return int(age) // width
+
+
+def wls_log_linear_fit(ages: np.ndarray, mean_mass: np.ndarray, weights: np.ndarray):
+    """Eq. 6: fit log Abar_r(dt) ~ log c_r - lambda_r dt by weighted least
+    squares, weights = observation counts (the count-weighted fit of
+    Sec. IV-B).  Normal equations of min sum w (y - a - b x)^2 with
+    x = age, y = log mean mass.  Returns (lambda_hat, log c_hat)."""
+    x = np.asarray(ages, np.float64)
+    y = np.log(np.asarray(mean_mass, np.float64))
+    w = np.asarray(weights, np.float64)
+    W, Sx, Sy = w.sum(), (w * x).sum(), (w * y).sum()
+    Sxx, Sxy = (w * x * x).sum(), (w * x * y).sum()
+    slope = (W * Sxy - Sx * Sy) / (W * Sxx - Sx * Sx)
+    intercept = (Sy - slope * Sx) / W
+    return -slope, intercept
+
+
+def half_life(rate: float) -> float:
+    """Eq. 7: t_half = ln 2 / lambda."""
+    return math.log(2.0) / rate if rate > 0 else math.inf
+
+
+def calibrate(mass_sum: np.ndarray, count: np.ndarray, width: int = CALIB_BUCKET_WIDTH,
+              min_count: int = 1):
+    """Per region: the mean attention mass of each age bucket (bucket centre
+    age width*b + width/2, as Fig. 3 plots), then the Eq. 6 fit over the
+    buckets with at least min_count observations and a positive mean.
+    Returns (lambda_hat[r], half_life[r]); NaN where fewer than two buckets."""
+    R, NB = mass_sum.shape
+    rates = np.full(R, np.nan)
+    halves = np.full(R, np.nan)
+    for r in range(R):
+        ok = (count[r] >= max(1, min_count)) & (mass_sum[r] > 0)
+        if ok.sum() < 2:
+            continue
+        b = np.nonzero(ok)[0]
+        ages = width * b + width / 2.0
+        lam, _ = wls_log_linear_fit(ages, mass_sum[r, b] / count[r, b], count[r, b])
+        rates[r] = lam
+        halves[r] = half_life(lam)
+    return rates, halves
+
+
 # ------------------------------------------------------------------ state ---
 @dataclass
 class OracleConfig:
@@ -171,6 +221,18 @@ class Oracle:
         self.base = np.zeros(NUM_REGIONS)
         self.half_life = np.full(NUM_REGIONS, np.inf)
         self.pinned = np.zeros(NUM_REGIONS, bool)
+        # calibration (Sec. IV-B): insertion step per slot, histogram of the
+        # observed mass by (region, age bucket)
+        self.t_ins = np.zeros(nslots, np.int64)
+        self.calib_on = False
+        self.calib_sum = np.zeros((NUM_REGIONS, CALIB_BUCKETS))
+        self.calib_cnt = np.zeros((NUM_REGIONS, CALIB_BUCKETS), np.int64)
+
+    def calib_enable(self, on: bool = True) -> None:
+        """Start (and clear) or stop gathering the calibration histogram."""
+        self.calib_on = bool(on)
+        self.calib_sum[:] = 0.0
+        self.calib_cnt[:] = 0
 
     # -- configuration (Table 1: base priority, decay rate, pinned flag) --
     def set_region_params(self, r: int, base: float, half_life: float, pinned: bool) -> None:
@@ -203,6 +265,7 @@ class Oracle:
         slot = phys * ps + off
         self.region[slot] = region
         self.t_ref[slot] = insert_step
+        self.t_ins[slot] = insert_step
         self.a[slot] = 0.0
         self.W[slot] = 0.0
         self.abar[slot] = 0.0
@@ -286,6 +349,12 @@ class Oracle:
             tau = c.tau_scale / n
             self.t_ref[sl] = refresh(self.t_ref[sl], abar, tau, self.t)
             self.W[sl] = 0.0
+            if self.calib_on:
+                for i, slot in enumerate(sl):
+                    bkt = age_bucket(self.t - self.t_ins[slot])
+                    if 0 <= bkt < CALIB_BUCKETS:
+                        self.calib_sum[reg[i], bkt] += abar[i]
+                        self.calib_cnt[reg[i], bkt] += 1
         d = decay(self.t - self.t_ref[sl], self.half_life[reg])
         s = token_score(self.base[reg], d, self.a[sl], c.attn_weight, c.score_mode)
         pinned_tok = self.pinned[reg]

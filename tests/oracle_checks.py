@@ -370,10 +370,65 @@ def check_bf16_widening(om):
     assert list(got) == want
 
 
+# ------------------------------------------------------------ calibration ---
+def check_calibration_fit(om):
+    """Eq. 6-7: on exactly exponential bucket means the count-weighted fit
+    returns the true rate and half-life; with noise it agrees with numpy's
+    least-squares routine (an independent implementation: SVD-based lstsq on
+    the sqrt-weighted system)."""
+    ages = np.arange(0, 160, 4) + 2.0
+    for lam in (0.002, 0.0217, 0.0495):     # half-lives ~347, 32, 14 steps (Table 2 range)
+        mean = 0.013 * np.exp(-lam * ages)
+        cnt = np.arange(len(ages), 0, -1) * 7
+        got, logc = om.wls_log_linear_fit(ages, mean, cnt)
+        assert abs(got - lam) < 1e-12 and abs(logc - math.log(0.013)) < 1e-10
+        assert abs(om.half_life(got) - math.log(2) / lam) < 1e-8
+    rng = np.random.default_rng(23)
+    mean = 0.01 * np.exp(-0.03 * ages) * np.exp(rng.normal(0, 0.2, len(ages)))
+    cnt = rng.integers(1, 500, len(ages))
+    lam, logc = om.wls_log_linear_fit(ages, mean, cnt)
+    sw = np.sqrt(cnt)
+    A = np.stack([np.ones_like(ages), ages], axis=1) * sw[:, None]
+    coef = np.linalg.lstsq(A, np.log(mean) * sw, rcond=None)[0]
+    assert abs(lam + coef[1]) < 1e-12 and abs(logc - coef[0]) < 1e-12
+    # calibrate(): bucket centres width*b + width/2, regions with < 2 buckets -> NaN
+    S = np.zeros((7, 8))
+    C = np.zeros((7, 8), np.int64)
+    C[2, :5] = 10
+    S[2, :5] = 10 * 0.02 * np.exp(-0.05 * (4 * np.arange(5) + 2))
+    C[3, 1] = 4
+    S[3, 1] = 0.1
+    rates, halves = om.calibrate(S, C)
+    assert abs(rates[2] - 0.05) < 1e-12 and np.isnan(rates[3]) and np.isnan(rates[0])
+
+
+def check_calibration_histogram(om):
+    """The histogram gathers Abar by (region, age // 4): with identical keys
+    every token gets Abar = 1/|K_t| exactly, so each bucket's sum is its
+    count / |K_t|, with ages counted from the insertion steps."""
+    o = make(om, L=1, Hq=2, Hkv=1, D=16, ps=4, phys=32)
+    regions = np.array([1] * 5 + [4] * 6, np.uint8)
+    steps = np.array([-9, -9, -9, -1, -1, -5, -5, -5, -5, -30, -30])
+    K, V = zeros_kv(1, 1, len(regions), 16)
+    o.append_tokens(0, regions, K, V, steps)
+    o.calib_enable(True)
+    zq = np.zeros((1, 1, 2, 16), np.uint16)
+    zkv = np.zeros((1, 1, 1, 16), np.uint16)
+    o.decode_step(1, zq, zkv, zkv, [6])           # t = 1: ages 10,10,10,2,2 | 6 x4, 31, 31 | new 0
+    o.evict(1, [100])
+    n = 12
+    want = {(1, 2): 3, (1, 0): 2, (4, 1): 4, (4, 7): 2, (6, 0): 1}
+    for (r, b), c in want.items():
+        assert o.calib_cnt[r, b] == c, (r, b, o.calib_cnt[r, b])
+        assert abs(o.calib_sum[r, b] - c / n) < 1e-15
+    assert o.calib_cnt.sum() == n
+
+
 ALL_CHECKS = [
     check_decay_closed_forms, check_fig2_trajectories, check_ewma_closed_form,
     check_attention_closed_form, check_mass_sums_to_one, check_gqa_mapping,
     check_refresh_threshold, check_page_scores, check_selection_bruteforce,
     check_token_level_objective, check_compaction_and_conservation,
     check_over_budget_and_no_observation, check_bf16_widening,
+    check_calibration_fit, check_calibration_histogram,
 ]

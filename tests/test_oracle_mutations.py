@@ -52,6 +52,10 @@ MUTANTS = {
     "attention_transposed_values": ("attention_group", _attn_transposed_values),
     "select_max_heap": ("select_pages_min_heap", lambda S, ev, k: sorted(
         sorted([p for p in range(len(S)) if ev[p]], key=lambda p: (-float(S[p]), p))[:k])),
+    "fit_unweighted": ("wls_log_linear_fit", lambda x, y, w, f=om.wls_log_linear_fit: f(x, y, np.ones_like(np.asarray(w, float)))),
+    "fit_wrong_sign": ("wls_log_linear_fit", lambda x, y, w, f=om.wls_log_linear_fit: (-f(x, y, w)[0], f(x, y, w)[1])),
+    "bucket_width_8": ("age_bucket", lambda age, width=4: int(age) // 8),
+    "half_life_without_ln2": ("half_life", lambda rate: 1.0 / rate if rate > 0 else math.inf),
     "select_ignores_pins": ("select_pages_min_heap", lambda S, ev, k: sorted(
         sorted(range(len(S)), key=lambda p: (float(S[p]), p))[:k])),
 }

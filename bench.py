@@ -54,6 +54,8 @@ def parse():
                     help="truncate every trace to this many tokens (small profiling cases)")
     ap.add_argument("--layerwise", action="store_true",
                     help="decode through md_decode_layer, one call per layer")
+    ap.add_argument("--calib", action="store_true",
+                    help="gather the calibration histogram (Eqs. 6-7) during observation steps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -227,6 +229,8 @@ def run_native(args, rank, world, local_rank):
         if cache.query(md.MD_QUERY_WINDOW) > 0:
             cache.evict(budgets)
         torch.cuda.synchronize()
+    if args.calib:
+        cache.calib_enable(True)
     saved = cache.save_state()
     tokens_step = sum(cache.query(md.MD_QUERY_TOKENS, b) + 1 for b in range(B))
     restore = args.phase == "full"
@@ -382,7 +386,8 @@ def workload_config(w, args):
             else "steady state",
             "l2": "no flush: inputs larger than L2 (K/V read per step >> 129 MB)",
             "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed,
-            "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict"}
+            "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict",
+            "calibration_histogram": bool(args.calib)}
 
 
 def combine_over_ranks(total_ms: float, tokens_total: float, device):

@@ -79,6 +79,8 @@ enum {
 #define MD_MAX_GROUP 8            /* query heads per KV head (GQA group)      */
 #define MD_MAX_CHUNKS 64          /* attention splits per (seq, layer, head)  */
 #define MD_MAX_CHUNK_TOKENS 4096  /* tokens per attention split               */
+#define MD_CALIB_BUCKETS 256      /* age buckets of the calibration histogram  */
+#define MD_CALIB_BUCKET_WIDTH 4   /* decode steps per age bucket (Fig. 3)      */
 
 typedef struct {
   /* Geometry: L layers, Hq query heads, Hkv KV heads (Hq / Hkv <= 8), head_dim
@@ -202,7 +204,8 @@ enum {
   MD_STATE_REGION = 7,      /* uint8 [slots] region label                             */
   MD_STATE_WINDOW = 8,      /* fp32  [slots] attention mass of folded window steps    */
   MD_STATE_MASS = 9,        /* fp32  [L*Hkv][slots] mass rows of the last decode step */
-  MD_STATE_POOL = 10        /* bf16  [L][num_phys_pages][Hkv][2][page_size][D] K/V    */
+  MD_STATE_POOL = 10,       /* bf16  [L][num_phys_pages][Hkv][2][page_size][D] K/V    */
+  MD_STATE_T_INS = 11       /* int32 [slots] insertion step                           */
 };
 
 /* Device-to-device copy of one state array into dst_dev (bytes must equal the
@@ -264,6 +267,34 @@ md_status md_debug_set(md_ctx *ctx, int key, int64_t value);
 
 /* Text of the last error on this handle ("" if none). */
 const char *md_last_error(const md_ctx *ctx);
+
+/* ---- calibration by-product (Sec. IV-B, Eqs. 6-7) --------------------- */
+
+/* While enabled, every observation step (md_evict after decode steps) adds
+ * each cached token's observed mass Abar_i to a histogram indexed by its
+ * region and its age bucket floor((t - t_ins) / MD_CALIB_BUCKET_WIDTH), ages
+ * 0 .. MD_CALIB_BUCKETS * width - 1 (older tokens are not counted): the data
+ * behind the paper's per-region lifetime curves (Fig. 3).  Enabling clears
+ * the histogram.  Sums are kept in fixed point (resolution 2^-32 per token),
+ * so the histogram is deterministic. */
+md_status md_calib_enable(md_ctx *ctx, int enable);
+
+/* Copies the histogram out: mass_sum[r][b] (sum of Abar), count[r][b]
+ * (observations), r < MD_NUM_REGIONS, b < MD_CALIB_BUCKETS (host arrays).
+ * Synchronises the handle's stream. */
+md_status md_calib_read(md_ctx *ctx, double *mass_sum, int64_t *count);
+
+/* Eq. 6 fit, host arithmetic only: per region, over the buckets with at least
+ * min_count observations and a positive mean, weighted least squares of
+ * log(mean mass) against the bucket's centre age (bucket_width * b +
+ * bucket_width / 2) with the observation counts as weights (the count-weighted
+ * fit of Sec. IV-B).  rate_out[r] = lambda_hat_r (NaN with fewer than two
+ * buckets), half_life_out[r] = ln 2 / lambda_hat_r (Eq. 7; +inf if
+ * lambda_hat_r <= 0).  Arrays are [MD_NUM_REGIONS][n_buckets] in,
+ * [MD_NUM_REGIONS] out. */
+md_status md_calib_fit(const double *mass_sum, const int64_t *count, int n_buckets,
+                       int bucket_width, int64_t min_count, double *rate_out,
+                       double *half_life_out);
 
 /* ---- stage 1 for callers that cannot allocate device memory ----------- */
 

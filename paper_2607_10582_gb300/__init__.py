@@ -36,7 +36,10 @@ MD_MAX_BATCH = 256
 MD_HEAD_DIM = 128
 
 (MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A, MD_STATE_T_REF,
- MD_STATE_AHAT, MD_STATE_FREE, MD_STATE_REGION, MD_STATE_WINDOW, MD_STATE_MASS, MD_STATE_POOL) = range(11)
+ MD_STATE_AHAT, MD_STATE_FREE, MD_STATE_REGION, MD_STATE_WINDOW, MD_STATE_MASS, MD_STATE_POOL,
+ MD_STATE_T_INS) = range(12)
+MD_CALIB_BUCKETS = 256
+MD_CALIB_BUCKET_WIDTH = 4
 (MD_QUERY_TOKENS, MD_QUERY_PAGES, MD_QUERY_FREE_TOP, MD_QUERY_STEP, MD_QUERY_WINDOW,
  MD_QUERY_PINNED_PAGES) = range(6)
 (MD_DEBUG_SPIN_LIMIT_NS, MD_DEBUG_EXTRA_ARRIVALS, MD_DEBUG_GRID_LIMIT, MD_DEBUG_UNIT_OVERHEAD,
@@ -79,6 +82,9 @@ SIGNATURES = {
     "md_profile_enable": (_c.c_int, [_P, _c.c_int]),
     "md_profile_read": (_c.c_int, [_P, _P, _P, _c.c_int]),
     "md_debug_set": (_c.c_int, [_P, _c.c_int, _c.c_int64]),
+    "md_calib_enable": (_c.c_int, [_P, _c.c_int]),
+    "md_calib_read": (_c.c_int, [_P, _P, _P]),
+    "md_calib_fit": (_c.c_int, [_P, _P, _c.c_int, _c.c_int, _c.c_int64, _P, _P]),
     "md_last_error": (_c.c_char_p, [_P]),
     "md_attend_mass_noalloc": (_c.c_int, [_P, _P, _P, _P, _P, _P, _c.c_int, _c.c_int, _c.c_int, _c.c_int,
                                           _c.c_int, _c.c_int, _c.c_int, _P]),
@@ -126,6 +132,20 @@ def _host(arr, dtype):
 
 def md_workspace_size(cfg: md_config) -> int:
     return int(lib().md_workspace_size(ctypes.byref(cfg)))
+
+
+def md_calib_fit(mass_sum: np.ndarray, count: np.ndarray, bucket_width: int = MD_CALIB_BUCKET_WIDTH,
+                 min_count: int = 1):
+    """Eq. 6-7 fit of a calibration histogram: (rate[7], half_life[7])."""
+    s = np.ascontiguousarray(mass_sum, np.float64)
+    n = np.ascontiguousarray(count, np.int64)
+    rate = np.zeros(MD_NUM_REGIONS)
+    half = np.zeros(MD_NUM_REGIONS)
+    st = lib().md_calib_fit(s.ctypes.data, n.ctypes.data, s.shape[1], bucket_width, min_count,
+                            rate.ctypes.data, half.ctypes.data)
+    if st != MD_OK:
+        raise MemDecayError(st, "md_calib_fit")
+    return rate, half
 
 
 class Cache:
@@ -231,6 +251,7 @@ class Cache:
             MD_STATE_WINDOW: ((slots,), t.float32),
             MD_STATE_MASS: ((self.L * self.Hkv, slots), t.float32),
             MD_STATE_POOL: ((self.L, self.P_phys, self.Hkv, 2, self.ps, MD_HEAD_DIM), t.int16),
+            MD_STATE_T_INS: ((slots,), t.int32),
         }[what]
 
     def get_state(self, what: int):
@@ -266,6 +287,16 @@ class Cache:
         n = np.zeros(5, np.int64)
         self._check(lib().md_profile_read(self.h, ms.ctypes.data, n.ctypes.data, 5))
         return {STAGES[i]: (float(ms[i]), int(n[i])) for i in range(5)}
+
+    def calib_enable(self, on: bool = True):
+        self._check(lib().md_calib_enable(self.h, int(on)))
+
+    def calib_read(self):
+        """(mass_sum [7][256], count [7][256]) of the calibration histogram."""
+        s = np.zeros((MD_NUM_REGIONS, MD_CALIB_BUCKETS), np.float64)
+        n = np.zeros((MD_NUM_REGIONS, MD_CALIB_BUCKETS), np.int64)
+        self._check(lib().md_calib_read(self.h, s.ctypes.data, n.ctypes.data))
+        return s, n
 
     def debug_set(self, key: int, value: int):
         self._check(lib().md_debug_set(self.h, key, value))

@@ -65,6 +65,7 @@ struct md_ctx {
   int grid_cap = 0;          // 0: every CTA that fits
   int unit_overhead = 4;     // planner: per-unit cost in pages
   int force_chunks = 0;      // planner: 0 = choose
+  bool calib_on = false;     // calibration histogram being gathered
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
   std::vector<ProfRec> pending;
@@ -310,6 +311,7 @@ size_t md::compute_layout(const md_config &c, Layout *lay) {
   L.region = take(L.slots, 256);
   L.a = take(L.slots * 4, 256);
   L.t_ref = take(L.slots * 4, 256);
+  L.t_ins = take(L.slots * 4, 256);
   L.window = take(L.slots * 4, 256);
   L.ahat = take(L.slots * 4, 256);
   L.prio = take(L.slots * 4, 256);
@@ -320,6 +322,7 @@ size_t md::compute_layout(const md_config &c, Layout *lay) {
   L.evict_list = take((size_t)c.max_batch * c.max_pages_per_seq * 4, 256);
   L.staging_regions = take((size_t)c.max_pages_per_seq * ps, 256);
   L.staging_steps = take((size_t)c.max_pages_per_seq * ps * 4, 256);
+  L.calib = take((size_t)8 * CALIB_BUCKETS * (8 + 4), 256);
   L.total = align_up(off, 256);
   if (lay) *lay = L;
   return L.total;
@@ -469,6 +472,7 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
   ap.ahat = ptr<float>(c, c->lay.ahat);
   ap.prio = ptr<float>(c, c->lay.prio);
   ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
+  ap.t_ins = ptr<int32_t>(c, c->lay.t_ins);
   ap.k_src = (const uint16_t *)k_dev;
   ap.v_src = (const uint16_t *)v_dev;
   ap.sb = 0;
@@ -536,6 +540,7 @@ void fill_append_common(md_ctx *c, AppendParams &ap) {
   ap.ahat = ptr<float>(c, c->lay.ahat);
   ap.prio = ptr<float>(c, c->lay.prio);
   ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
+  ap.t_ins = ptr<int32_t>(c, c->lay.t_ins);
   ap.Hkv = cf.num_kv_heads;
   ap.ps = cf.page_size;
   ap.P_phys = cf.num_phys_pages;
@@ -729,8 +734,12 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   sp.prio = ptr<float>(c, c->lay.prio);
   sp.page_score = ptr<float>(c, c->lay.page_score);
   sp.t_ref = ptr<int32_t>(c, c->lay.t_ref);
+  sp.t_ins = ptr<int32_t>(c, c->lay.t_ins);
   sp.region = ptr<uint8_t>(c, c->lay.region);
   sp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  sp.calib_sum = ptr<unsigned long long>(c, c->lay.calib);
+  sp.calib_cnt = (unsigned int *)(c->ws + c->lay.calib + (size_t)8 * CALIB_BUCKETS * 8);
+  sp.calib_on = c->calib_on ? 1 : 0;
   sp.slots = (long long)c->lay.slots;
   sp.rows = cf.num_layers * cf.num_kv_heads;
   sp.ps = ps;
@@ -856,6 +865,7 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
       *off = L.mass;
       *bytes = (size_t)cf.num_layers * cf.num_kv_heads * L.slots * 4;
       return true;
+    case MD_STATE_T_INS: *off = L.t_ins; *bytes = L.slots * 4; return true;
     case MD_STATE_POOL:
       *off = L.pool;
       *bytes = (size_t)cf.num_layers * cf.num_phys_pages * cf.num_kv_heads * 2 * cf.page_size * D * 2;
@@ -865,7 +875,7 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
 }
 const int SAVED[] = {MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A,
                      MD_STATE_T_REF,       MD_STATE_AHAT,       MD_STATE_FREE,       MD_STATE_REGION,
-                     MD_STATE_WINDOW};
+                     MD_STATE_WINDOW,      MD_STATE_T_INS};
 }  // namespace
 
 MD_API md_status md_get_state(md_ctx *c, int what, void *dst, size_t bytes) {
@@ -1039,6 +1049,71 @@ MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
     return MD_OK;
   }
   return fail(c, MD_ERR_INVALID_ARG, "unknown debug key");
+}
+
+MD_API md_status md_calib_enable(md_ctx *c, int enable) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  c->calib_on = enable != 0;
+  if (c->calib_on) {
+    cudaError_t e = cudaMemsetAsync(c->ws + c->lay.calib, 0, (size_t)8 * CALIB_BUCKETS * 12, c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "calibration clear");
+  }
+  return MD_OK;
+}
+
+MD_API md_status md_calib_read(md_ctx *c, double *mass_sum, int64_t *count) {
+  if (!c || !mass_sum || !count) return MD_ERR_INVALID_ARG;
+  std::vector<unsigned long long> s((size_t)8 * CALIB_BUCKETS);
+  std::vector<unsigned int> n((size_t)8 * CALIB_BUCKETS);
+  cudaError_t e = cudaMemcpyAsync(s.data(), c->ws + c->lay.calib, s.size() * 8, cudaMemcpyDeviceToHost,
+                                  c->stream);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(n.data(), c->ws + c->lay.calib + s.size() * 8, n.size() * 4,
+                        cudaMemcpyDeviceToHost, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "calibration read");
+  for (int r = 0; r < MD_NUM_REGIONS; ++r)
+    for (int b = 0; b < CALIB_BUCKETS; ++b) {
+      const size_t k = (size_t)r * CALIB_BUCKETS + b;
+      mass_sum[k] = (double)s[k] * (1.0 / 4294967296.0);
+      count[k] = n[k];
+    }
+  return MD_OK;
+}
+
+MD_API md_status md_calib_fit(const double *mass_sum, const int64_t *count, int n_buckets,
+                              int bucket_width, int64_t min_count, double *rate_out,
+                              double *half_life_out) {
+  if (!mass_sum || !count || !rate_out || !half_life_out || n_buckets < 1 || bucket_width < 1)
+    return MD_ERR_INVALID_ARG;
+  for (int r = 0; r < MD_NUM_REGIONS; ++r) {
+    /* weighted least squares of y = log(mean) on x = centre age, w = count */
+    double W = 0, Sx = 0, Sy = 0, Sxx = 0, Sxy = 0;
+    int used = 0;
+    for (int b = 0; b < n_buckets; ++b) {
+      const int64_t n = count[(size_t)r * n_buckets + b];
+      const double m = mass_sum[(size_t)r * n_buckets + b];
+      if (n < (min_count > 1 ? min_count : 1) || !(m > 0)) continue;
+      const double x = (double)bucket_width * b + 0.5 * bucket_width;
+      const double y = log(m / (double)n);
+      const double w = (double)n;
+      W += w;
+      Sx += w * x;
+      Sy += w * y;
+      Sxx += w * x * x;
+      Sxy += w * x * y;
+      ++used;
+    }
+    if (used < 2) {
+      rate_out[r] = NAN;
+      half_life_out[r] = NAN;
+      continue;
+    }
+    const double slope = (W * Sxy - Sx * Sy) / (W * Sxx - Sx * Sx);
+    rate_out[r] = -slope;
+    half_life_out[r] = rate_out[r] > 0 ? log(2.0) / rate_out[r] : INFINITY;
+  }
+  return MD_OK;
 }
 
 MD_API const char *md_last_error(const md_ctx *c) { return c ? c->err.c_str() : "null handle"; }

@@ -18,6 +18,8 @@ constexpr int PARTIAL_FLOATS = 1088;        // m[8] l[8] O[8][128], padded to 25
 constexpr int MAX_GRID = 512;               // persistent attention CTAs (>= 2 x SM count)
 
 enum DevStatus { ST_CODE = 0, ST_ABORT = 1, ST_DIAG = 2, ST_WORDS = 8 };
+constexpr int CALIB_BUCKETS = MD_CALIB_BUCKETS;      // age buckets per region
+constexpr int CALIB_WIDTH = MD_CALIB_BUCKET_WIDTH;   // decode steps per bucket
 
 struct RegionTable {
   float base[8];
@@ -27,8 +29,8 @@ struct RegionTable {
 
 /* Byte offsets of every array inside the caller's workspace. */
 struct Layout {
-  size_t pool, block_table, page_score, free_stack, region, a, t_ref, window, ahat, prio, mass,
-      scratch, partials, counters, evict_list, staging_regions, staging_steps, status, total;
+  size_t pool, block_table, page_score, free_stack, region, a, t_ref, t_ins, window, ahat, prio, mass,
+      scratch, partials, counters, evict_list, staging_regions, staging_steps, status, calib, total;
   size_t slots, n_items;
   int scratch_tokens, chunk_stride;
 };
@@ -42,7 +44,7 @@ struct AppendParams {
   const int32_t *free_stack;
   uint8_t *region;
   float *a, *window, *ahat, *prio;
-  int32_t *t_ref;
+  int32_t *t_ref, *t_ins;
   const uint16_t *k_src, *v_src;
   long long sb, sl, sh, si;              // element strides of the source (seq, layer, head, token)
   const uint8_t *regions_dev;            // per token (prefill) or null
@@ -93,8 +95,12 @@ struct ScoreParams {
   const float *mass;
   float *window, *a, *ahat, *prio, *page_score;
   int32_t *t_ref;
+  const int32_t *t_ins;
   const uint8_t *region;
   const int32_t *block_table;
+  unsigned long long *calib_sum;   // [8][CALIB_BUCKETS] observed mass, fixed point 2^-32
+  unsigned int *calib_cnt;         // [8][CALIB_BUCKETS] observations
+  int calib_on;
   long long slots;
   int rows, ps, P_max;
   int fold_only;         // 1: window += mass rows and nothing else

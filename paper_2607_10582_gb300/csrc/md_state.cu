@@ -78,6 +78,7 @@ __global__ void append_kernel(const __grid_constant__ AppendParams p) {
       const size_t slot = (size_t)phys * p.ps + off;
       p.region[slot] = p.regions_dev ? p.regions_dev[i] : p.regions_param[j];
       p.t_ref[slot] = p.steps_dev ? p.steps_dev[i] : p.insert_step;
+      p.t_ins[slot] = p.t_ref[slot];
       p.a[slot] = 0.f;
       p.window[slot] = 0.f;
       p.ahat[slot] = 0.f;
@@ -129,10 +130,22 @@ __device__ __forceinline__ float sum_rows(const float *mass, long long slots, in
 template <int PS>
 __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
   constexpr int PPW = 32 / PS;
+  /* calibration histogram of this block (Sec. IV-B, Eq. 6's input): observed
+   * mass in fixed point, so integer atomics keep the sums order-independent */
+  __shared__ unsigned long long h_sum[8 * CALIB_BUCKETS];
+  __shared__ unsigned int h_cnt[8 * CALIB_BUCKETS];
   const int lane = threadIdx.x & 31;
   const int warps_total = (gridDim.x * blockDim.x) >> 5;
   const int warp_id = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const float INF = INFINITY;
+  const bool calib = p.calib_on && p.observe && !p.fold_only;
+  if (calib) {
+    for (int k = threadIdx.x; k < 8 * CALIB_BUCKETS; k += blockDim.x) {
+      h_sum[k] = 0ull;
+      h_cnt[k] = 0u;
+    }
+    __syncthreads();
+  }
   for (int base = warp_id * PPW; base < p.total_pages; base += warps_total * PPW) {
     const int gp = base + lane / PS;
     const int off = lane % PS;
@@ -167,6 +180,14 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
           p.ahat[slot] = abar;
           p.a[slot] = a;
           p.t_ref[slot] = tr;
+          if (calib) {
+            const int age = p.t - p.t_ins[slot];
+            const int bkt = age >= 0 ? age / CALIB_WIDTH : -1;
+            if (bkt >= 0 && bkt < CALIB_BUCKETS) {
+              atomicAdd(&h_sum[reg * CALIB_BUCKETS + bkt], __float2ull_rn(abar * 4294967296.0f));
+              atomicAdd(&h_cnt[reg * CALIB_BUCKETS + bkt], 1u);
+            }
+          }
         }
         const float x = __fdiv_rn((float)(p.t - tr), p.reg.half_life[reg]);
         const float d = exp2f(-x);                                    // Eqs. 4, 7
@@ -196,6 +217,14 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
         p.page_score[(size_t)b * p.P_max + pg] = S;
       }
     }
+  }
+  if (calib) {
+    __syncthreads();
+    for (int k = threadIdx.x; k < 8 * CALIB_BUCKETS; k += blockDim.x)
+      if (h_cnt[k]) {
+        atomicAdd(&p.calib_sum[k], h_sum[k]);
+        atomicAdd(&p.calib_cnt[k], h_cnt[k]);
+      }
   }
 }
 

@@ -48,7 +48,7 @@ def rel_err(g, o):
 
 
 class Lockstep:
-    def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2, layerwise=False):
+    def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2, layerwise=False, calib=False):
         self.w = w
         self.layerwise = layerwise
         B = w.B
@@ -62,6 +62,9 @@ class Lockstep:
         for r in range(7):
             self.gpu.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
             self.orc.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+        if calib:
+            self.gpu.calib_enable(True)
+            self.orc.calib_enable(True)
         self.pos = [0] * B
         self.step_no = 0
         self.resyncs = {"evict": 0, "refresh": 0}
@@ -210,6 +213,21 @@ class Lockstep:
         free[:len(o.free)] = o.free
         self.gpu.set_state(md.MD_STATE_BLOCK_TABLE, torch.from_numpy(bt).cuda())
         self.gpu.set_state(md.MD_STATE_FREE, torch.from_numpy(free).cuda())
+
+    def check_calibration(self):
+        """Histogram counts bit-exact, mass sums within the Abar tolerance (plus
+        the 2^-33 fixed-point rounding per observation), Eq. 6 rates close."""
+        gs, gc = self.gpu.calib_read()
+        o = self.orc
+        assert np.array_equal(gc, o.calib_cnt), "calibration counts differ"
+        tol = TOL_REL * np.abs(o.calib_sum) + gc * 2.0 ** -32 + TOL_FLOOR
+        assert np.all(np.abs(gs - o.calib_sum) <= tol), "calibration sums differ"
+        rate, _ = md.md_calib_fit(gs, gc)
+        orate, _ = om.calibrate(o.calib_sum, o.calib_cnt)
+        assert np.array_equal(np.isnan(rate), np.isnan(orate))
+        ok = ~np.isnan(orate)
+        assert np.all(np.abs(rate[ok] - orate[ok]) <= 1e-3 * np.abs(orate[ok]) + 1e-6), (rate, orate)
+        return gc.sum()
 
     def check_layout(self):
         """Block tables and free stack bit-exact against the oracle."""

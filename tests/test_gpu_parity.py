@@ -129,6 +129,20 @@ def test_layer_by_layer_call_order_is_enforced():
     assert c.sync() == md.MD_OK
 
 
+def test_calibration_histogram_and_fit():
+    """The calibration by-product (Sec. IV-B, Eqs. 6-7): the region x age
+    histogram of the observed mass, gathered on the GPU during observation
+    steps, matches the oracle's, and so do the fitted rates."""
+    w = synth.custom_workload("calib", L=2, Hq=16, Hkv=2, page_size=16, lengths=[1200, 700],
+                              budget_frac=0.6, steps=24, seed=14, structured=True)
+    w.insert_steps[0][:] = -np.arange(1200)[::-1] // 3      # a spread of ages
+    ls = Lockstep(w, calib=True).run()
+    assert ls.check_calibration() > 1000
+    w3 = synth.custom_workload("calib_win", L=2, Hq=8, Hkv=2, page_size=32, lengths=[900],
+                               budget_frac=0.5, steps=12, seed=15, window_k=4)
+    Lockstep(w3, calib=True).run().check_calibration()
+
+
 def test_config1_first_steps():
     """Config 1 geometry (Qwen2.5-1.5B, 28 layers, 12/2 heads), 1,700 tokens."""
     ls = Lockstep(synth.make_workload(1))

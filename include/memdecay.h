@@ -94,6 +94,15 @@ typedef struct {
    *   refresh when Abar_i >= tau_scale / |K_t|                 (Eq. 3)
    *   score_mode 0: s_i = b_r 2^(-dt/h_r) + attn_weight a_i    (Eq. 4)
    *   score_mode 1: s_i = (b_r + attn_weight a_i) 2^(-dt/h_r)
+   *   score_mode 2: s_i = b_r 2^(-dt/h_r) + attn_weight a_i |K_t|: the
+   *                 attention term relative to the uniform level 1/|K_t|, the
+   *                 change the paper's ablation points to (Sec. IV-D, Sec. V)
+   *   score_mode 3: s_i = t_ins_i (recency; the streaming baseline, Sec. IV-C)
+   *   score_mode 4: s_i = uniform draw per token and observation step from
+   *                 random_seed (the random baseline, Sec. IV-C)
+   *   (the H2O-style baseline of Sec. IV-C is score_mode 0 with rho = gamma
+   *    = 1, every b_r = 0 and no pinned region: accumulated attention)
+   *   Pinned regions score +inf in every mode.
    *   page_reduce 0: S_p = mean over the page's tokens (Eq. 5); 1: max. */
   float rho, gamma, tau_scale, attn_weight;
   int score_mode, page_reduce;
@@ -101,6 +110,7 @@ typedef struct {
   void *workspace;            /* device memory, 256-byte aligned, caller-owned */
   size_t workspace_bytes;
   void *stream;               /* cudaStream_t (NULL = legacy default stream) */
+  uint64_t random_seed;       /* score_mode 4 only */
 } md_config;
 
 /* Bytes of device workspace md_create needs for cfg (0 if cfg is invalid).

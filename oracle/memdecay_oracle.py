@@ -99,12 +99,42 @@ def decay(dt: np.ndarray, half_life: np.ndarray) -> np.ndarray:
     return np.power(2.0, -(dt / h))
 
 
-def token_score(base: np.ndarray, d: np.ndarray, a: np.ndarray, alpha: float, mode: int) -> np.ndarray:
-    """Eq. 4: s_i = b_r d_i + alpha a_i (mode 0, the paper's additive form);
-    mode 1 is the multiplicative reading (b_r + alpha a_i) d_i."""
+def token_score(base: np.ndarray, d: np.ndarray, a: np.ndarray, alpha: float, mode: int,
+                n_cached: int = 1, t_ins: np.ndarray = None, noise: np.ndarray = None) -> np.ndarray:
+    """Retention score of each token.
+    mode 0: Eq. 4, s_i = b_r d_i + alpha a_i (the paper's additive form);
+    mode 1: the multiplicative reading (b_r + alpha a_i) d_i;
+    mode 2: Eq. 4 with the attention term normalised to the uniform level
+            1/|K_t| (the design change of Sec. IV-D / Sec. V): b_r d_i + alpha a_i |K_t|;
+    mode 3: recency (the streaming baseline of Sec. IV-C): newer tokens score
+            higher, s_i = t_ins_i;
+    mode 4: a uniform random draw per token and observation (the random
+            baseline of Sec. IV-C)."""
     if mode == 0:
         return base * d + alpha * a
-    return (base + alpha * a) * d
+    if mode == 1:
+        return (base + alpha * a) * d
+    if mode == 2:
+        return base * d + alpha * a * float(n_cached)
+    if mode == 3:
+        return np.asarray(t_ins, np.float64)
+    return np.asarray(noise, np.float64)
+
+
+def random_draw(seed: int, t: int, slot: np.ndarray) -> np.ndarray:
+    """Uniform draws in [0, 1) for the random baseline: the SplitMix64
+    finaliser (Steele, Lea, Flood 2014) of (seed, step, physical slot), top 24
+    bits scaled by 2^-24 (exact in fp32)."""
+    M = (1 << 64) - 1
+    out = np.empty(len(slot))
+    for i, sl in enumerate(np.asarray(slot, np.int64)):
+        x = ((seed * 0x9E3779B97F4A7C15) ^ (int(t) << 40) ^ int(sl)) & M
+        z = (x + 0x9E3779B97F4A7C15) & M
+        z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & M
+        z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & M
+        z = z ^ (z >> 31)
+        out[i] = (z >> 40) * 2.0 ** -24
+    return out
 
 
 def page_score(member_scores: np.ndarray, reduce_mode: int) -> float:
@@ -194,6 +224,7 @@ class OracleConfig:
     attn_weight: float = 1.0
     score_mode: int = 0
     page_reduce: int = 0
+    random_seed: int = 0
 
 
 class Oracle:
@@ -356,7 +387,9 @@ class Oracle:
                         self.calib_sum[reg[i], bkt] += abar[i]
                         self.calib_cnt[reg[i], bkt] += 1
         d = decay(self.t - self.t_ref[sl], self.half_life[reg])
-        s = token_score(self.base[reg], d, self.a[sl], c.attn_weight, c.score_mode)
+        noise = random_draw(c.random_seed, self.t, sl) if c.score_mode == 4 else None
+        s = token_score(self.base[reg], d, self.a[sl], c.attn_weight, c.score_mode, n,
+                        self.t_ins[sl], noise)
         pinned_tok = self.pinned[reg]
         s = np.where(pinned_tok, np.inf, s)
         self.prio[sl] = s

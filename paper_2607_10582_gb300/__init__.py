@@ -57,6 +57,7 @@ class md_config(ctypes.Structure):
         ("score_mode", ctypes.c_int), ("page_reduce", ctypes.c_int), ("keep_token_prio", ctypes.c_int),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
         ("stream", ctypes.c_void_p),
+        ("random_seed", ctypes.c_uint64),
     ]
 
 
@@ -156,7 +157,7 @@ class Cache:
                  max_batch: int, max_pages_per_seq: int, num_phys_pages: int, *,
                  rho: float = 0.9, gamma: float = 0.1, tau_scale: float = 2.0,
                  attn_weight: float = 1.0, score_mode: int = 0, page_reduce: int = 0,
-                 keep_token_prio: int = 1, stream=None, device=None):
+                 keep_token_prio: int = 1, random_seed: int = 0, stream=None, device=None):
         import torch
         self.torch = torch
         self.device = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
@@ -164,7 +165,7 @@ class Cache:
         c = md_config(num_layers, num_q_heads, num_kv_heads, MD_HEAD_DIM, page_size,
                       max_batch, max_pages_per_seq, num_phys_pages,
                       rho, gamma, tau_scale, attn_weight, score_mode, page_reduce, keep_token_prio,
-                      None, 0, ctypes.c_void_p(self.stream.cuda_stream))
+                      None, 0, ctypes.c_void_p(self.stream.cuda_stream), random_seed)
         need = md_workspace_size(c)
         if need == 0:
             raise MemDecayError(MD_ERR_INVALID_ARG, "invalid configuration")

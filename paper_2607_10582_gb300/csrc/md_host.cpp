@@ -120,7 +120,7 @@ const char *check_config(const md_config &c) {
     return "rho must be in [0,1] and gamma >= 0";
   if (!(c.tau_scale >= 0.f) || !isfinite(c.tau_scale)) return "tau_scale must be >= 0";
   if (!(c.attn_weight >= 0.f) || !isfinite(c.attn_weight)) return "attn_weight must be >= 0";
-  if (c.score_mode != 0 && c.score_mode != 1) return "score_mode must be 0 or 1";
+  if (c.score_mode < 0 || c.score_mode > 4) return "score_mode must be in [0, 4]";
   if (c.page_reduce != 0 && c.page_reduce != 1) return "page_reduce must be 0 or 1";
   return nullptr;
 }
@@ -754,6 +754,7 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   sp.tau_scale = cf.tau_scale;
   sp.alpha = cf.attn_weight;
   sp.score_mode = cf.score_mode;
+  sp.random_seed = cf.random_seed;
   sp.page_reduce = cf.page_reduce;
   sp.keep_prio = 1;
   sp.reg = c->reg;

@@ -109,6 +109,7 @@ struct ScoreParams {
   int t;
   float rho, gamma, tau_scale, alpha;
   int score_mode, page_reduce, keep_prio;
+  unsigned long long random_seed;
   RegionTable reg;
   int n_seqs, total_pages;
   int n_tokens[MD_MAX_BATCH];

@@ -107,6 +107,19 @@ __device__ __forceinline__ int find_seq(const int *start, int n, int x) {
   return lo;
 }
 
+/* Uniform draw in [0, 1) for the random-baseline score: the SplitMix64
+ * finaliser (Steele, Lea and Flood, 2014) of (seed, step, slot); the top 24
+ * bits scaled by 2^-24 are exact in fp32. */
+__device__ __forceinline__ float random_draw(unsigned long long seed, int t, size_t slot) {
+  unsigned long long z = (seed * 0x9E3779B97F4A7C15ull) ^ ((unsigned long long)(unsigned)t << 40) ^
+                         (unsigned long long)slot;
+  z += 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  z ^= z >> 31;
+  return (float)(z >> 40) * 5.9604644775390625e-08f;
+}
+
 /* Sum of one token's mass over the rows (layer, KV head) in a fixed order,
  * four partial sums so that many row loads are in flight per lane. */
 __device__ __forceinline__ float sum_rows(const float *mass, long long slots, int rows, size_t slot) {
@@ -191,8 +204,13 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
         }
         const float x = __fdiv_rn((float)(p.t - tr), p.reg.half_life[reg]);
         const float d = exp2f(-x);                                    // Eqs. 4, 7
-        s = (p.score_mode == 0) ? p.reg.base[reg] * d + p.alpha * a
-                                : (p.reg.base[reg] + p.alpha * a) * d;
+        switch (p.score_mode) {
+          case 0: s = p.reg.base[reg] * d + p.alpha * a; break;       // Eq. 4
+          case 1: s = (p.reg.base[reg] + p.alpha * a) * d; break;
+          case 2: s = p.reg.base[reg] * d + p.alpha * a * (float)p.n_tokens[b]; break;
+          case 3: s = (float)p.t_ins[slot]; break;                     // recency
+          default: s = random_draw(p.random_seed, p.t, slot); break;   // random
+        }
         pinned = p.reg.pinned[reg];
         if (pinned) s = INF;
         if (p.keep_prio) p.prio[slot] = s;

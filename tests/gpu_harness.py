@@ -55,7 +55,8 @@ class Lockstep:
         self.P_max = w.max_pages_per_seq()
         self.P_phys = w.num_phys_pages() + phys_slack
         kw = dict(rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
-                  score_mode=w.score_mode, page_reduce=w.page_reduce)
+                  score_mode=w.score_mode, page_reduce=w.page_reduce,
+                  random_seed=w.extra.get("random_seed", 0))
         self.gpu = md.Cache(w.L, w.Hq, w.Hkv, w.page_size, B, self.P_max, self.P_phys, **kw)
         self.orc = om.Oracle(om.OracleConfig(w.L, w.Hq, w.Hkv, w.D, w.page_size, B, self.P_max,
                                              self.P_phys, **kw))

@@ -424,11 +424,42 @@ def check_calibration_histogram(om):
     assert o.calib_cnt.sum() == n
 
 
+# --------------------------------------------------------- policy variants ---
+def check_policy_variants(om):
+    """Mode 2 (attention term relative to the uniform level 1/|K_t|): under
+    uniform attention a_1 = gamma/|K_t|, so alpha a |K_t| = alpha gamma for any
+    |K_t|.  Mode 3 (recency) evicts the oldest evictable pages first, as a
+    streaming window does.  Mode 4 draws are uniform in [0, 1): their mean and
+    spread over many draws match U(0,1), and they are reproducible."""
+    for n0 in (9, 30):
+        o = make(om, L=1, Hq=2, Hkv=1, D=16, ps=4, phys=32, score_mode=2, attn_weight=3.0)
+        K, V = zeros_kv(1, 1, n0, 16)
+        o.append_tokens(0, np.full(n0, 2, np.uint8), K, V, 0)
+        z = np.zeros((1, 1, 2, 16), np.uint16)
+        zk = np.zeros((1, 1, 1, 16), np.uint16)
+        o.decode_step(1, z, zk, zk, [2])
+        o.evict(1, [100])
+        s0 = o.prio[o.slots(0)[0]]
+        assert abs(s0 - (0.5 * 2 ** (-1 / 30) + 3.0 * 0.1)) < 1e-12, (n0, s0)
+    o = make(om, L=1, Hq=2, Hkv=1, D=16, ps=4, phys=32, score_mode=3)
+    K, V = zeros_kv(1, 1, 24, 16)
+    o.append_tokens(0, np.full(24, 3, np.uint8), K, V, np.repeat(np.arange(-6, 0), 4))
+    z = np.zeros((1, 1, 2, 16), np.uint16)
+    zk = np.zeros((1, 1, 1, 16), np.uint16)
+    o.decode_step(1, z, zk, zk, [3])
+    st, n, ids, logical = o.evict(1, [4])
+    assert logical[0] == [0, 1, 2], logical
+    u = om.random_draw(5, 3, np.arange(20000))
+    assert 0.0 <= u.min() and u.max() < 1.0 and abs(u.mean() - 0.5) < 0.01 and abs(u.var() - 1 / 12) < 0.003
+    assert np.array_equal(u, om.random_draw(5, 3, np.arange(20000)))
+    assert not np.array_equal(u, om.random_draw(5, 4, np.arange(20000)))
+
+
 ALL_CHECKS = [
     check_decay_closed_forms, check_fig2_trajectories, check_ewma_closed_form,
     check_attention_closed_form, check_mass_sums_to_one, check_gqa_mapping,
     check_refresh_threshold, check_page_scores, check_selection_bruteforce,
     check_token_level_objective, check_compaction_and_conservation,
     check_over_budget_and_no_observation, check_bf16_widening,
-    check_calibration_fit, check_calibration_histogram,
+    check_calibration_fit, check_calibration_histogram, check_policy_variants,
 ]

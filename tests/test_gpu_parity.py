@@ -83,6 +83,24 @@ def test_score_variants(score_mode, page_reduce, w):
     Lockstep(wl).run().check_layout()
 
 
+@pytest.mark.parametrize("mode", [2, 3, 4])
+def test_policy_variants(mode):
+    """Score modes beyond Eq. 4: the attention term normalised to the uniform
+    level (2), recency / streaming (3), seeded random (4), and the H2O-style
+    accumulated-attention configuration (mode 0, rho = gamma = 1, b = 0)."""
+    w = synth.custom_workload("pol", L=2, Hq=16, Hkv=2, page_size=16, lengths=[900, 1500],
+                              budget_frac=0.3, steps=8, seed=16, score_mode=mode, structured=True)
+    for b in range(w.B):
+        w.insert_steps[b][:] = -(np.arange(w.n0(b))[::-1] // 16)
+    w.extra["random_seed"] = 99
+    Lockstep(w).run().check_layout()
+    if mode == 2:
+        h2o = synth.custom_workload("h2o", L=2, Hq=16, Hkv=2, page_size=16, lengths=[1100],
+                                    budget_frac=0.3, steps=8, seed=17, rho=1.0, gamma=1.0,
+                                    base=(0.0,) * 7, pinned=(0,) * 7, structured=True)
+        Lockstep(h2o).run().check_layout()
+
+
 def test_pins_over_budget_warns():
     """Pinned pages alone exceed the budget: every evictable page goes, the
     warning comes back, pinned pages stay."""

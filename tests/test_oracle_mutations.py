@@ -42,8 +42,12 @@ MUTANTS = {
     "refresh_strict": ("refresh", lambda t_ref, abar, tau, t:
                        np.where(np.asarray(abar, np.float32) > np.float32(tau), t, t_ref)),
     "refresh_never": ("refresh", lambda t_ref, abar, tau, t: t_ref),
-    "score_dropped_attention": ("token_score", lambda base, d, a, alpha, mode: base * d),
-    "score_dropped_decay": ("token_score", lambda base, d, a, alpha, mode: base + alpha * a),
+    "score_dropped_attention": ("token_score", lambda base, d, a, alpha, mode, *r: base * d),
+    "score_dropped_decay": ("token_score", lambda base, d, a, alpha, mode, *r: base + alpha * a),
+    "normalised_term_unscaled": ("token_score", lambda base, d, a, alpha, mode, n=1, ti=None, nz=None,
+                                 f=om.token_score: f(base, d, a, alpha, 0 if mode == 2 else mode, n, ti, nz)),
+    "recency_reversed": ("token_score", lambda base, d, a, alpha, mode, n=1, ti=None, nz=None,
+                         f=om.token_score: -np.asarray(ti, float) if mode == 3 else f(base, d, a, alpha, mode, n, ti, nz)),
     "page_sum_not_mean": ("page_score", lambda s, mode: float(np.sum(s))),
     "page_min_not_mean": ("page_score", lambda s, mode: float(np.min(s))),
     "mass_wrong_divisor": ("observed_mass", lambda W, k, L, Hq: W / float(k * L)),

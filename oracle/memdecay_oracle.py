@@ -225,6 +225,7 @@ class OracleConfig:
     score_mode: int = 0
     page_reduce: int = 0
     random_seed: int = 0
+    region_aligned: bool = False
 
 
 class Oracle:
@@ -239,6 +240,8 @@ class Oracle:
         # LIFO free stack of physical page ids; the first pop returns 0.
         self.free: List[int] = list(range(cfg.num_phys_pages - 1, -1, -1))
         self.block: List[List[int]] = [[] for _ in range(cfg.max_batch)]
+        self.fill: List[List[int]] = [[] for _ in range(cfg.max_batch)]   # tokens per page
+        self.tail_region = [-1] * cfg.max_batch
         self.n_tokens = [0] * cfg.max_batch
         nslots = cfg.num_phys_pages * ps
         self.region = np.zeros(nslots, np.uint8)
@@ -282,13 +285,20 @@ class Oracle:
     def _append_one(self, b: int, region: int, k: np.ndarray, v: np.ndarray, insert_step: int) -> None:
         """Append one token (Fig. 1 "append KV"): region label r(i), insertion
         step t_ins, clock t_ref = t_ins, importance a = 0.  A full (or absent)
-        tail page takes a fresh physical page from the free stack."""
+        tail page takes a fresh physical page from the free stack; with
+        region-aligned allocation (the variant Sec. III-D leaves to future
+        work) a token whose region differs from the tail page's also opens a
+        fresh page, so no page straddles a region boundary."""
         ps = self.cfg.page_size
-        off = self.n_tokens[b] % ps
-        if off == 0:
+        fills = self.fill[b]
+        if not fills or fills[-1] == ps or (self.cfg.region_aligned and self.tail_region[b] != region):
             if len(self.block[b]) >= self.cfg.max_pages_per_seq or not self.free:
                 raise RuntimeError("capacity")
             self.block[b].append(self.free.pop())
+            fills.append(0)
+        off = fills[-1]
+        fills[-1] += 1
+        self.tail_region[b] = region
         phys = self.block[b][-1]
         kp, vp = self._page(phys)
         kp[:, :, off, :] = k
@@ -318,17 +328,18 @@ class Oracle:
             self._append_one(b, int(regions[i]), K[:, :, i, :], V[:, :, i, :], int(steps[i]))
 
     def slots(self, b: int) -> np.ndarray:
-        """Physical slots of sequence b in logical order."""
+        """Physical slots of sequence b's tokens in logical order."""
         ps = self.cfg.page_size
-        n = self.n_tokens[b]
-        return np.array([self.block[b][i // ps] * ps + i % ps for i in range(n)], np.int64)
+        return np.array([phys * ps + o for phys, f in zip(self.block[b], self.fill[b]) for o in range(f)],
+                        np.int64)
+
+    def page_of_token(self, b: int) -> np.ndarray:
+        """Logical page index of each of sequence b's tokens (logical order)."""
+        return np.repeat(np.arange(len(self.fill[b])), self.fill[b])
 
     def _gather(self, b: int, l: int, h: int) -> Tuple[np.ndarray, np.ndarray]:
-        ps = self.cfg.page_size
-        n = self.n_tokens[b]
         ks, vs = [], []
-        for j, phys in enumerate(self.block[b]):
-            cnt = min(ps, n - j * ps)
+        for phys, cnt in zip(self.block[b], self.fill[b]):
             kp, vp = self.pool[phys]
             ks.append(kp[l, h, :cnt])
             vs.append(vp[l, h, :cnt])
@@ -395,8 +406,9 @@ class Oracle:
         self.prio[sl] = s
         P = len(self.block[b])
         S = np.zeros(P)
+        bounds = np.concatenate([[0], np.cumsum(self.fill[b])])
         for j in range(P):
-            lo, hi = j * ps, min(n, (j + 1) * ps)
+            lo, hi = bounds[j], bounds[j + 1]
             if pinned_tok[lo:hi].any() or j == P - 1:      # pinning / protected tail
                 S[j] = np.inf
             else:
@@ -424,10 +436,11 @@ class Oracle:
             if sum(evictable) < want:
                 status = MD_WARN_OVER_BUDGET
             out = select_pages_min_heap(S32, evictable, want)
+            gone = set(out)
             freed = [self.block[b][j] for j in out]
-            keep = [self.block[b][j] for j in range(P) if j not in set(out)]
-            self.block[b] = keep
-            self.n_tokens[b] -= len(out) * self.cfg.page_size
+            self.n_tokens[b] -= sum(self.fill[b][j] for j in out)
+            self.block[b] = [self.block[b][j] for j in range(P) if j not in gone]
+            self.fill[b] = [self.fill[b][j] for j in range(P) if j not in gone]
             n_ev.append(len(out))
             ids.append(freed)
             logical.append(out)

@@ -455,6 +455,48 @@ def check_policy_variants(om):
     assert not np.array_equal(u, om.random_draw(5, 4, np.arange(20000)))
 
 
+# -------------------------------------------------- region-aligned pages ---
+def check_region_aligned_pages(om):
+    """Region-aligned allocation (Sec. III-D: a fresh page at each region
+    boundary) leaves no page straddling a boundary; pages keep their partial
+    fill, eviction removes exactly their tokens, and on page-aligned spans it
+    makes the same layout as the default allocator."""
+    regions = np.array([0] * 5 + [1] * 7 + [2] * 3 + [1] * 9, np.uint8)
+    for aligned in (False, True):
+        o = make(om, L=1, Hq=2, Hkv=1, D=16, ps=4, phys=32, region_aligned=aligned)
+        K, V = zeros_kv(1, 1, len(regions), 16)
+        o.append_tokens(0, regions, K, V, 0)
+        sl = o.slots(0)
+        pages = o.page_of_token(0)
+        straddle = sum(len(set(regions[pages == p])) > 1 for p in range(len(o.block[0])))
+        if aligned:
+            assert o.fill[0] == [4, 1, 4, 3, 3, 4, 4, 1] and straddle == 0
+        else:
+            assert o.fill[0] == [4] * 6 and straddle == 2
+        assert len(sl) == len(regions) and o.n_tokens[0] == len(regions)
+        assert np.array_equal(o.region[sl], regions)
+    # eviction removes the evicted pages' tokens, whatever their fill
+    o = make(om, L=1, Hq=2, Hkv=1, D=16, ps=4, phys=32, region_aligned=True)
+    for r in range(7):
+        o.set_region_params(r, 0.1 * (r + 1), 30.0, False)
+    K, V = zeros_kv(1, 1, len(regions), 16)
+    o.append_tokens(0, regions, K, V, 0)
+    z = np.zeros((1, 1, 2, 16), np.uint16)
+    zk = np.zeros((1, 1, 1, 16), np.uint16)
+    o.decode_step(1, z, zk, zk, [1])           # region 1 joins the last region-1 page
+    st, n, ids, logical = o.evict(1, [6])
+    assert o.fill[0][-1] == 2 and logical[0] == [0, 1]
+    assert o.n_tokens[0] == len(regions) + 1 - 5
+    # page-aligned spans: identical layout with or without alignment
+    r2 = np.array([3] * 8 + [5] * 4 + [6] * 12, np.uint8)
+    outs = []
+    for aligned in (False, True):
+        o = make(om, L=1, Hq=2, Hkv=1, D=16, ps=4, phys=32, region_aligned=aligned)
+        o.append_tokens(0, r2, *zeros_kv(1, 1, len(r2), 16), 0)
+        outs.append((list(o.block[0]), list(o.fill[0]), list(o.slots(0))))
+    assert outs[0] == outs[1]
+
+
 ALL_CHECKS = [
     check_decay_closed_forms, check_fig2_trajectories, check_ewma_closed_form,
     check_attention_closed_form, check_mass_sums_to_one, check_gqa_mapping,
@@ -462,4 +504,5 @@ ALL_CHECKS = [
     check_token_level_objective, check_compaction_and_conservation,
     check_over_budget_and_no_observation, check_bf16_widening,
     check_calibration_fit, check_calibration_histogram, check_policy_variants,
+    check_region_aligned_pages,
 ]

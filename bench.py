@@ -54,6 +54,8 @@ def parse():
                     help="truncate every trace to this many tokens (small profiling cases)")
     ap.add_argument("--layerwise", action="store_true",
                     help="decode through md_decode_layer, one call per layer")
+    ap.add_argument("--aligned", action="store_true",
+                    help="region-aligned page allocation (a fresh page at each region boundary)")
     ap.add_argument("--calib", action="store_true",
                     help="gather the calibration histogram (Eqs. 6-7) during observation steps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -167,9 +169,15 @@ def run_native(args, rank, world, local_rank):
     stream = torch.cuda.current_stream(dev)
     w = make_workload(args, args.seed + rank)
     B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
-    cache = md.Cache(L, Hq, Hkv, ps, B, w.max_pages_per_seq(), w.num_phys_pages(),
+    P_max, P_phys = w.max_pages_per_seq(), w.num_phys_pages()
+    if args.aligned:   # each region span can leave one partly filled page
+        spans = [int(np.count_nonzero(np.diff(w.regions[b].astype(np.int16)))) + 1 for b in range(B)]
+        P_max += max(spans)
+        P_phys += sum(spans)
+    cache = md.Cache(L, Hq, Hkv, ps, B, P_max, P_phys,
                      rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
-                     score_mode=w.score_mode, page_reduce=w.page_reduce, keep_token_prio=0)
+                     score_mode=w.score_mode, page_reduce=w.page_reduce, keep_token_prio=0,
+                     region_aligned_pages=int(args.aligned))
     for r in range(7):
         cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
     lib = synth.lib()
@@ -387,7 +395,8 @@ def workload_config(w, args):
             "l2": "no flush: inputs larger than L2 (K/V read per step >> 129 MB)",
             "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed,
             "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict",
-            "calibration_histogram": bool(args.calib)}
+            "calibration_histogram": bool(args.calib),
+            "page_allocation": "region-aligned" if args.aligned else "contiguous"}
 
 
 def combine_over_ranks(total_ms: float, tokens_total: float, device):

@@ -111,6 +111,11 @@ typedef struct {
   size_t workspace_bytes;
   void *stream;               /* cudaStream_t (NULL = legacy default stream) */
   uint64_t random_seed;       /* score_mode 4 only */
+  /* 1: region-aligned page allocation -- a token whose region differs from
+   * the page being written opens a fresh page, so no page holds two regions
+   * (the allocator variant Sec. III-D leaves to future work).  Pages may then
+   * be partly filled; every stage masks by each page's fill. */
+  int region_aligned_pages;
 } md_config;
 
 /* Bytes of device workspace md_create needs for cfg (0 if cfg is invalid).
@@ -215,7 +220,9 @@ enum {
   MD_STATE_WINDOW = 8,      /* fp32  [slots] attention mass of folded window steps    */
   MD_STATE_MASS = 9,        /* fp32  [L*Hkv][slots] mass rows of the last decode step */
   MD_STATE_POOL = 10,       /* bf16  [L][num_phys_pages][Hkv][2][page_size][D] K/V    */
-  MD_STATE_T_INS = 11       /* int32 [slots] insertion step                           */
+  MD_STATE_T_INS = 11,      /* int32 [slots] insertion step                           */
+  MD_STATE_PAGE_FILL = 12,  /* uint8 [max_batch][max_pages_per_seq] tokens per page   */
+  MD_STATE_SEQ_TOKENS = 13  /* int32 [max_batch] tokens per sequence (device count)   */
 };
 
 /* Device-to-device copy of one state array into dst_dev (bytes must equal the
@@ -224,8 +231,8 @@ md_status md_get_state(md_ctx *ctx, int what, void *dst_dev, size_t bytes);
 
 /* Overwrites one state array from src_dev (test support: lets a parity test
  * put the oracle's choice back where floating-point ties allowed the GPU
- * another valid one).  Only BLOCK_TABLE, FREE, A and T_REF; the caller keeps
- * the array consistent with the host mirror's counts. */
+ * another valid one).  Only BLOCK_TABLE, FREE, A, T_REF, PAGE_FILL and
+ * SEQ_TOKENS; the caller keeps them consistent with the host mirror's counts. */
 md_status md_set_state(md_ctx *ctx, int what, const void *src_dev, size_t bytes);
 
 enum {

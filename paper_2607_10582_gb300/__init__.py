@@ -37,7 +37,7 @@ MD_HEAD_DIM = 128
 
 (MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A, MD_STATE_T_REF,
  MD_STATE_AHAT, MD_STATE_FREE, MD_STATE_REGION, MD_STATE_WINDOW, MD_STATE_MASS, MD_STATE_POOL,
- MD_STATE_T_INS) = range(12)
+ MD_STATE_T_INS, MD_STATE_PAGE_FILL, MD_STATE_SEQ_TOKENS) = range(14)
 MD_CALIB_BUCKETS = 256
 MD_CALIB_BUCKET_WIDTH = 4
 (MD_QUERY_TOKENS, MD_QUERY_PAGES, MD_QUERY_FREE_TOP, MD_QUERY_STEP, MD_QUERY_WINDOW,
@@ -58,6 +58,7 @@ class md_config(ctypes.Structure):
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
         ("stream", ctypes.c_void_p),
         ("random_seed", ctypes.c_uint64),
+        ("region_aligned_pages", ctypes.c_int),
     ]
 
 
@@ -157,7 +158,8 @@ class Cache:
                  max_batch: int, max_pages_per_seq: int, num_phys_pages: int, *,
                  rho: float = 0.9, gamma: float = 0.1, tau_scale: float = 2.0,
                  attn_weight: float = 1.0, score_mode: int = 0, page_reduce: int = 0,
-                 keep_token_prio: int = 1, random_seed: int = 0, stream=None, device=None):
+                 keep_token_prio: int = 1, random_seed: int = 0, region_aligned_pages: int = 0,
+                 stream=None, device=None):
         import torch
         self.torch = torch
         self.device = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
@@ -165,7 +167,8 @@ class Cache:
         c = md_config(num_layers, num_q_heads, num_kv_heads, MD_HEAD_DIM, page_size,
                       max_batch, max_pages_per_seq, num_phys_pages,
                       rho, gamma, tau_scale, attn_weight, score_mode, page_reduce, keep_token_prio,
-                      None, 0, ctypes.c_void_p(self.stream.cuda_stream), random_seed)
+                      None, 0, ctypes.c_void_p(self.stream.cuda_stream), random_seed,
+                      int(region_aligned_pages))
         need = md_workspace_size(c)
         if need == 0:
             raise MemDecayError(MD_ERR_INVALID_ARG, "invalid configuration")
@@ -253,6 +256,8 @@ class Cache:
             MD_STATE_MASS: ((self.L * self.Hkv, slots), t.float32),
             MD_STATE_POOL: ((self.L, self.P_phys, self.Hkv, 2, self.ps, MD_HEAD_DIM), t.int16),
             MD_STATE_T_INS: ((slots,), t.int32),
+            MD_STATE_PAGE_FILL: ((self.max_batch, self.P_max), t.uint8),
+            MD_STATE_SEQ_TOKENS: ((self.max_batch,), t.int32),
         }[what]
 
     def get_state(self, what: int):

@@ -49,7 +49,7 @@ struct AttnShape {
   static constexpr int MERGE_FLOATS = NCW * (24 + GP * D);
   static constexpr int FIN_FLOATS = 16 + 3 * MD_MAX_CHUNKS * GP;
   static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * Q_BYTES + (2 * R + 4) * 8 +
-                                 4 * MERGE_FLOATS + 4 * FIN_FLOATS + 4 * MAX_UNIT_PAGES + 64;
+                                 4 * MERGE_FLOATS + 4 * FIN_FLOATS + 8 * MAX_UNIT_PAGES + 4 * R + 64;
 };
 
 struct Unit {
@@ -108,7 +108,9 @@ __device__ __forceinline__ uint32_t swz(uint32_t stage, int row, int d) {
   return stage + half * (2 * PS * 128) + row * 128 + ((chunk ^ (row & 7)) << 4);
 }
 
-template <int PS, int NCW>
+/* ALIGNED: pages carry their own fill (region-aligned allocation); otherwise
+ * every page but the last is full and the fills follow from n_tokens. */
+template <int PS, int NCW, bool ALIGNED>
 __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW>::CTAS_PER_SM)
     attn_mass_kernel(const __grid_constant__ AttnParams p,
                      const __grid_constant__ CUtensorMap tmap) {
@@ -130,7 +132,9 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   float *pl = pm + MD_MAX_CHUNKS * GP;        // [MD_MAX_CHUNKS][8] partial sums
   float *fac = pl + MD_MAX_CHUNKS * GP;       // [MD_MAX_CHUNKS][8] combine factors
   int *sphys = (int *)(fac + MD_MAX_CHUNKS * GP);   // [MAX_UNIT_PAGES] page ids
-  int *flag = sphys + S::MAX_UNIT_PAGES;
+  int *sfill = sphys + S::MAX_UNIT_PAGES;            // [MAX_UNIT_PAGES] tokens per page
+  int *fillbuf = sfill + S::MAX_UNIT_PAGES;          // [R] fill of the page in each stage
+  int *flag = fillbuf + S::R;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -178,9 +182,14 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
         const int32_t *bt = p.block_table + (size_t)un.b * p.P_max;
         for (int pb = un.p0; pb < un.p1 && ok; pb += 8) {
           const int cnt = min(8, un.p1 - pb);
-          int ph[8];
+          int ph[8], fl[8];
 #pragma unroll
           for (int k = 0; k < 8; ++k) ph[k] = k < cnt ? bt[pb + k] : 0;
+          if (ALIGNED) {
+            const uint8_t *fr = p.page_fill + (size_t)un.b * p.P_max;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) fl[k] = k < cnt ? fr[pb + k] : 0;
+          }
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             if (k >= cnt) break;
@@ -192,6 +201,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
             }
             const int row = (((un.l * p.P_phys + ph[k]) * p.Hkv + un.kvh) * 2) * PS;
             const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
+            if (ALIGNED) fillbuf[s] = fl[k];   // published by the arrive below
             mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
             tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
             tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
@@ -253,7 +263,10 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       pm[idx] = __ldcg(pj + (idx & 7));
       pl[idx] = __ldcg(pj + 8 + (idx & 7));
     }
-    for (int k = ct; k < pv.p1 - pv.p0; k += NC) sphys[k] = bt[pv.p0 + k];
+    for (int k = ct; k < pv.p1 - pv.p0; k += NC) {
+      sphys[k] = bt[pv.p0 + k];
+      if (ALIGNED) sfill[k] = p.page_fill[(size_t)pv.b * p.P_max + pv.p0 + k];
+    }
     named_barrier(1, NC);
     if (cw == 0) {
       /* per head: global max and normaliser over the C chunks */
@@ -305,7 +318,6 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     {
       const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + pv_slot) * p.scratch_tokens * GP;
       const int ntok = (pv.p1 - pv.p0) * PS;
-      const int nvalid = min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
       float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
       float fm[GP], fz[GP];
 #pragma unroll
@@ -313,8 +325,12 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
         fm[h] = fin[h];
         fz[h] = (h < G) ? fin[8 + h] : 0.f;
       }
+      /* contiguous pages: the valid tokens are a prefix of the unit; with
+       * region-aligned pages every page has its own fill */
+      const int nvalid = ALIGNED ? ntok : min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
 #pragma unroll 4
       for (int tk = ct; tk < nvalid; tk += NC) {
+        if (ALIGNED && (tk % PS) >= sfill[tk / PS]) continue;
         const float4 s0 = __ldcg((const float4 *)(scr + (size_t)tk * GP));
         const float4 s1 = __ldcg((const float4 *)(scr + (size_t)tk * GP + 4));
         float m = exp2f(s0.x - fm[0]) * fz[0] + exp2f(s0.y - fm[1]) * fz[1] +
@@ -374,7 +390,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
         break;
       }
       const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
-      const int fill = ntok_seq - (un.p0 + jp) * PS;
+      const int fill = ALIGNED ? fillbuf[s] : ntok_seq - (un.p0 + jp) * PS;
 
       float acc[S::NT][4];
 #pragma unroll
@@ -509,9 +525,9 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   if (!stopped && have_prev) finish(prev, (nunit - 1) & 1);
 }
 
-template <int PS, int NCW>
+template <int PS, int NCW, bool AL>
 static cudaError_t prepare_impl() {
-  return cudaFuncSetAttribute(attn_mass_kernel<PS, NCW>,
+  return cudaFuncSetAttribute(attn_mass_kernel<PS, NCW, AL>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)AttnShape<PS, NCW>::SMEM);
 }
@@ -521,8 +537,9 @@ static int grid_limit_impl() {
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-  if (prepare_impl<PS, NCW>() != cudaSuccess) return 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_mass_kernel<PS, NCW>,
+  if (prepare_impl<PS, NCW, false>() != cudaSuccess || prepare_impl<PS, NCW, true>() != cudaSuccess)
+    return 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_mass_kernel<PS, NCW, false>,
                                                     AttnShape<PS, NCW>::THREADS,
                                                     AttnShape<PS, NCW>::SMEM) != cudaSuccess)
     return 0;
@@ -530,7 +547,7 @@ static int grid_limit_impl() {
   return g > MAX_GRID ? MAX_GRID : g;
 }
 
-template <int PS, int NCW>
+template <int PS, int NCW, bool AL>
 static cudaError_t launch_impl(const AttnParams &p, const CUtensorMap &tmap, int grid,
                                cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
@@ -543,13 +560,15 @@ static cudaError_t launch_impl(const AttnParams &p, const CUtensorMap &tmap, int
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, attn_mass_kernel<PS, NCW>, p, tmap);
+  return cudaLaunchKernelEx(&cfg, attn_mass_kernel<PS, NCW, AL>, p, tmap);
 }
 
 constexpr int NCW_DEFAULT = 4;
 
 cudaError_t attention_prepare(int ps) {
-  return ps == 16 ? prepare_impl<16, NCW_DEFAULT>() : prepare_impl<32, NCW_DEFAULT>();
+  cudaError_t e = ps == 16 ? prepare_impl<16, NCW_DEFAULT, false>() : prepare_impl<32, NCW_DEFAULT, false>();
+  if (e != cudaSuccess) return e;
+  return ps == 16 ? prepare_impl<16, NCW_DEFAULT, true>() : prepare_impl<32, NCW_DEFAULT, true>();
 }
 
 int attention_grid_limit(int ps) {
@@ -559,8 +578,11 @@ int attention_grid_limit(int ps) {
 cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &tmap, int grid,
                              cudaStream_t s) {
   if (p.total_units == 0) return cudaSuccess;
-  return p.ps == 16 ? launch_impl<16, NCW_DEFAULT>(p, tmap, grid, s)
-                    : launch_impl<32, NCW_DEFAULT>(p, tmap, grid, s);
+  if (p.page_fill)
+    return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, true>(p, tmap, grid, s)
+                      : launch_impl<32, NCW_DEFAULT, true>(p, tmap, grid, s);
+  return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, false>(p, tmap, grid, s)
+                    : launch_impl<32, NCW_DEFAULT, false>(p, tmap, grid, s);
 }
 
 }  // namespace md

@@ -55,9 +55,10 @@ struct md_ctx {
   int grid_limit = 0;
   RegionTable reg;
   HostMirror m;
-  std::vector<int64_t> n_tokens;
+  std::vector<int64_t> n_tokens;           // tokens per sequence (exact while tokens_exact)
   std::vector<int> n_pages, pinned_pages;
-  std::vector<uint8_t> tail_pinned;
+  std::vector<int> tail_fill, tail_region;  // the page being written
+  std::vector<uint8_t> tail_pinned, tokens_exact;
   bool poisoned = false;
   std::string err;
   long long spin_limit_ns = 2000000000LL;
@@ -167,13 +168,29 @@ int evictable_pages(const md_ctx *c, int b) {
   return P - c->pinned_pages[b] - (c->tail_pinned[b] ? 0 : 1);
 }
 
-/* Pinned-page bookkeeping for one appended token of region r. */
-void mirror_token(md_ctx *c, int b, int r) {
+/* Whether a token of region r opens a fresh page: no page yet, the tail page
+ * full, or (region-aligned allocation) a region different from the tail's. */
+bool opens_page(const md_ctx *c, int b, int r) {
+  return c->n_pages[b] == 0 || c->tail_fill[b] == c->cfg.page_size ||
+         (c->cfg.region_aligned_pages && c->tail_region[b] != r);
+}
+
+/* Slot (page * page_size + offset, in logical page order) the next token of
+ * region r goes to. */
+int next_slot(const md_ctx *c, int b, int r) {
   const int ps = c->cfg.page_size;
-  if (c->n_tokens[b] % ps == 0) {
+  return opens_page(c, b, r) ? c->n_pages[b] * ps : (c->n_pages[b] - 1) * ps + c->tail_fill[b];
+}
+
+/* Mirror bookkeeping for one appended token of region r. */
+void mirror_token(md_ctx *c, int b, int r) {
+  if (opens_page(c, b, r)) {
     c->n_pages[b] += 1;
+    c->tail_fill[b] = 0;
     c->tail_pinned[b] = 0;
   }
+  c->tail_fill[b] += 1;
+  c->tail_region[b] = r;
   if (c->reg.pinned[r] && !c->tail_pinned[b]) {
     c->pinned_pages[b] += 1;
     c->tail_pinned[b] = 1;
@@ -183,7 +200,7 @@ void mirror_token(md_ctx *c, int b, int r) {
 
 int64_t cached_tokens(const md_ctx *c) {
   int64_t s = 0;
-  for (auto v : c->n_tokens) s += v;
+  for (auto v : c->n_pages) s += v;
   return s;
 }
 
@@ -196,6 +213,12 @@ md_status launch_fold(md_ctx *c) {
   sp.window = ptr<float>(c, c->lay.window);
   sp.region = ptr<uint8_t>(c, c->lay.region);
   sp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  /* with contiguous pages the host's exact counts describe every page; the
+   * device fills and counts are read only with region-aligned pages */
+  if (c->cfg.region_aligned_pages) {
+    sp.page_fill = ptr<uint8_t>(c, c->lay.page_fill);
+    sp.seq_tokens = ptr<int32_t>(c, c->lay.seq_tokens);
+  }
   sp.slots = (long long)c->lay.slots;
   sp.rows = c->cfg.num_layers * c->cfg.num_kv_heads;
   sp.ps = c->cfg.page_size;
@@ -322,6 +345,9 @@ size_t md::compute_layout(const md_config &c, Layout *lay) {
   L.evict_list = take((size_t)c.max_batch * c.max_pages_per_seq * 4, 256);
   L.staging_regions = take((size_t)c.max_pages_per_seq * ps, 256);
   L.staging_steps = take((size_t)c.max_pages_per_seq * ps * 4, 256);
+  L.staging_slots = take((size_t)c.max_pages_per_seq * ps * 4, 256);
+  L.page_fill = take((size_t)c.max_batch * c.max_pages_per_seq, 256);
+  L.seq_tokens = take((size_t)c.max_batch * 4, 256);
   L.calib = take((size_t)8 * CALIB_BUCKETS * (8 + 4), 256);
   L.total = align_up(off, 256);
   if (lay) *lay = L;
@@ -352,6 +378,9 @@ MD_API md_status md_create(const md_config *cfg, md_ctx **out) {
   c->n_pages.assign(B, 0);
   c->pinned_pages.assign(B, 0);
   c->tail_pinned.assign(B, 0);
+  c->tail_fill.assign(B, 0);
+  c->tail_region.assign(B, -1);
+  c->tokens_exact.assign(B, 1);
   for (int r = 0; r < 8; ++r) {
     c->reg.base[r] = 0.f;
     c->reg.half_life[r] = INFINITY;
@@ -442,8 +471,22 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
     for (int i = 0; i < n; ++i)
       if (steps_host[i] > c->m.t) return fail(c, MD_ERR_INVALID_ARG, "insertion step in the future");
   const int ps = cf.page_size;
-  const long long tok_after = c->n_tokens[seq] + (long long)n;
-  const long long pages_after = (tok_after + ps - 1) / ps;
+  /* where the tokens go: the same page-opening rule as the mirror */
+  std::vector<int32_t> slots(n);
+  long long pages_after = c->n_pages[seq];
+  {
+    int fill = c->tail_fill[seq], treg = c->tail_region[seq];
+    for (int i = 0; i < n; ++i) {
+      const int r = regions_host[i];
+      if (pages_after == 0 || fill == ps || (cf.region_aligned_pages && treg != r)) {
+        ++pages_after;
+        fill = 0;
+      }
+      slots[i] = (int32_t)((pages_after - 1) * ps + fill);
+      ++fill;
+      treg = r;
+    }
+  }
   const long long new_pages = pages_after - c->n_pages[seq];
   if (pages_after > cf.max_pages_per_seq)
     return fail(c, MD_ERR_CAPACITY, "sequence %d would need %lld pages (max %d)", seq,
@@ -460,6 +503,9 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
   if (e == cudaSuccess && steps_host)
     e = cudaMemcpyAsync(c->ws + c->lay.staging_steps, steps_host, (size_t)n * 4,
                         cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess && cf.region_aligned_pages)
+    e = cudaMemcpyAsync(c->ws + c->lay.staging_slots, slots.data(), (size_t)n * 4,
+                        cudaMemcpyHostToDevice, c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "staging copy");
   AppendParams ap;
   memset(&ap, 0, sizeof(ap));
@@ -473,6 +519,9 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
   ap.prio = ptr<float>(c, c->lay.prio);
   ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
   ap.t_ins = ptr<int32_t>(c, c->lay.t_ins);
+  ap.page_fill = ptr<uint8_t>(c, c->lay.page_fill);
+  ap.seq_tokens = ptr<int32_t>(c, c->lay.seq_tokens);
+  ap.slots_dev = cf.region_aligned_pages ? ptr<int32_t>(c, c->lay.staging_slots) : nullptr;
   ap.k_src = (const uint16_t *)k_dev;
   ap.v_src = (const uint16_t *)v_dev;
   ap.sb = 0;
@@ -493,7 +542,8 @@ MD_API md_status md_append_tokens(md_ctx *c, int seq, int n, const uint8_t *regi
   ap.n_per_seq = n;
   ap.seq0 = seq;
   ap.insert_step = (int)c->m.t;
-  ap.tok0[0] = (int)c->n_tokens[seq];
+  ap.tok0[0] = slots[0];
+  ap.pages_before[0] = c->n_pages[seq];
   ap.pop_base[0] = (int)(c->m.free_top - 1);
   cudaEvent_t e0;
   prof_begin(c, &e0);
@@ -518,7 +568,7 @@ md_status check_step(md_ctx *c, int batch, const uint8_t *new_region_host) {
   long long need_total = 0;
   for (int b = 0; b < batch; ++b) {
     if (!valid_region(new_region_host[b])) return fail(c, MD_ERR_INVALID_ARG, "bad region label");
-    const int need = (c->n_tokens[b] % ps == 0) ? 1 : 0;
+    const int need = opens_page(c, b, new_region_host[b]) ? 1 : 0;
     if (c->n_pages[b] + need > cf.max_pages_per_seq)
       return fail(c, MD_ERR_CAPACITY, "sequence %d block table full", b);
     need_total += need;
@@ -541,6 +591,8 @@ void fill_append_common(md_ctx *c, AppendParams &ap) {
   ap.prio = ptr<float>(c, c->lay.prio);
   ap.t_ref = ptr<int32_t>(c, c->lay.t_ref);
   ap.t_ins = ptr<int32_t>(c, c->lay.t_ins);
+  ap.page_fill = ptr<uint8_t>(c, c->lay.page_fill);
+  ap.seq_tokens = ptr<int32_t>(c, c->lay.seq_tokens);
   ap.Hkv = cf.num_kv_heads;
   ap.ps = cf.page_size;
   ap.P_phys = cf.num_phys_pages;
@@ -575,10 +627,11 @@ md_status begin_step(md_ctx *c, int batch, int l0, int L, long long sb, long lon
   ap.insert_step = (int)c->m.t;
   long long popped = 0;
   for (int b = 0; b < batch; ++b) {
-    ap.tok0[b] = (int)c->n_tokens[b];
+    ap.tok0[b] = next_slot(c, b, new_region_host[b]);
+    ap.pages_before[b] = c->n_pages[b];
     ap.pop_base[b] = (int)(c->m.free_top - 1 - popped);
     ap.regions_param[b] = new_region_host[b];
-    if (c->n_tokens[b] % ps == 0) popped += 1;
+    if (opens_page(c, b, new_region_host[b])) popped += 1;
   }
   cudaEvent_t e0;
   prof_begin(c, &e0);
@@ -599,6 +652,7 @@ md_status run_attention(md_ctx *c, int batch, int l0, int L, int q_layers, const
   atp.q = (const uint16_t *)q_dev;
   atp.out = (uint16_t *)out_dev;
   atp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  atp.page_fill = cf.region_aligned_pages ? ptr<uint8_t>(c, c->lay.page_fill) : nullptr;
   atp.mass = ptr<float>(c, c->lay.mass);
   atp.scratch = ptr<float>(c, c->lay.scratch);
   atp.partials = ptr<float>(c, c->lay.partials);
@@ -693,7 +747,8 @@ MD_API md_status md_decode_layer(md_ctx *c, int layer, int batch, const void *q_
     ap.init_state = 0;
     ap.lookup_only = 1;
     ap.n_seqs = batch;
-    for (int b = 0; b < batch; ++b) ap.tok0[b] = (int)c->n_tokens[b] - 1;
+    for (int b = 0; b < batch; ++b)
+      ap.tok0[b] = (c->n_pages[b] - 1) * cf.page_size + c->tail_fill[b] - 1;
     cudaEvent_t e0;
     prof_begin(c, &e0);
     cudaError_t e = launch_append(ap, c->stream);
@@ -737,6 +792,10 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   sp.t_ins = ptr<int32_t>(c, c->lay.t_ins);
   sp.region = ptr<uint8_t>(c, c->lay.region);
   sp.block_table = ptr<int32_t>(c, c->lay.block_table);
+  if (cf.region_aligned_pages) {
+    sp.page_fill = ptr<uint8_t>(c, c->lay.page_fill);
+    sp.seq_tokens = ptr<int32_t>(c, c->lay.seq_tokens);
+  }
   sp.calib_sum = ptr<unsigned long long>(c, c->lay.calib);
   sp.calib_cnt = (unsigned int *)(c->ws + c->lay.calib + (size_t)8 * CALIB_BUCKETS * 8);
   sp.calib_on = c->calib_on ? 1 : 0;
@@ -782,6 +841,8 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   sel.free_stack = ptr<int32_t>(c, c->lay.free_stack);
   sel.evict_list = ptr<int32_t>(c, c->lay.evict_list);
   sel.user_evicted = evicted_ids_dev;
+  sel.page_fill = ptr<uint8_t>(c, c->lay.page_fill);
+  sel.seq_tokens = ptr<int32_t>(c, c->lay.seq_tokens);
   sel.status = ptr<int>(c, c->lay.status);
   sel.P_max = cf.max_pages_per_seq;
   sel.n_seqs = batch;
@@ -809,7 +870,13 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   }
   for (int b = 0; b < batch; ++b) {
     c->n_pages[b] -= ev[b];
-    c->n_tokens[b] -= (int64_t)ev[b] * ps;
+    /* evicted pages are never the tail; they are full unless pages are
+     * region-aligned, where their fill is known on the device only */
+    if (cf.region_aligned_pages) {
+      if (ev[b] > 0) c->tokens_exact[b] = 0;
+    } else {
+      c->n_tokens[b] -= (int64_t)ev[b] * ps;
+    }
     if (n_evicted_host) n_evicted_host[b] = ev[b];
   }
   c->m.free_top += pushed;
@@ -867,6 +934,11 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
       *bytes = (size_t)cf.num_layers * cf.num_kv_heads * L.slots * 4;
       return true;
     case MD_STATE_T_INS: *off = L.t_ins; *bytes = L.slots * 4; return true;
+    case MD_STATE_PAGE_FILL:
+      *off = L.page_fill;
+      *bytes = (size_t)cf.max_batch * cf.max_pages_per_seq;
+      return true;
+    case MD_STATE_SEQ_TOKENS: *off = L.seq_tokens; *bytes = (size_t)cf.max_batch * 4; return true;
     case MD_STATE_POOL:
       *off = L.pool;
       *bytes = (size_t)cf.num_layers * cf.num_phys_pages * cf.num_kv_heads * 2 * cf.page_size * D * 2;
@@ -876,7 +948,7 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
 }
 const int SAVED[] = {MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A,
                      MD_STATE_T_REF,       MD_STATE_AHAT,       MD_STATE_FREE,       MD_STATE_REGION,
-                     MD_STATE_WINDOW,      MD_STATE_T_INS};
+                     MD_STATE_WINDOW,      MD_STATE_T_INS,      MD_STATE_PAGE_FILL,  MD_STATE_SEQ_TOKENS};
 }  // namespace
 
 MD_API md_status md_get_state(md_ctx *c, int what, void *dst, size_t bytes) {
@@ -891,7 +963,7 @@ MD_API md_status md_get_state(md_ctx *c, int what, void *dst, size_t bytes) {
 MD_API md_status md_set_state(md_ctx *c, int what, const void *src, size_t bytes) {
   if (!c || !src) return MD_ERR_INVALID_ARG;
   if (what != MD_STATE_BLOCK_TABLE && what != MD_STATE_FREE && what != MD_STATE_A &&
-      what != MD_STATE_T_REF)
+      what != MD_STATE_T_REF && what != MD_STATE_PAGE_FILL && what != MD_STATE_SEQ_TOKENS)
     return fail(c, MD_ERR_INVALID_ARG, "state array is read-only");
   size_t off, n;
   state_array(c, what, &off, &n);
@@ -905,7 +977,19 @@ MD_API md_status md_query(const md_ctx *c, int what, int seq, int64_t *out) {
   const bool per_seq = what == MD_QUERY_TOKENS || what == MD_QUERY_PAGES || what == MD_QUERY_PINNED_PAGES;
   if (per_seq && (seq < 0 || seq >= c->cfg.max_batch)) return MD_ERR_INVALID_ARG;
   switch (what) {
-    case MD_QUERY_TOKENS: *out = c->n_tokens[seq]; return MD_OK;
+    case MD_QUERY_TOKENS: {
+      if (c->tokens_exact[seq]) {
+        *out = c->n_tokens[seq];
+        return MD_OK;
+      }
+      int32_t v = 0;   /* region-aligned pages after an eviction: ask the device */
+      if (cudaStreamSynchronize(c->stream) != cudaSuccess ||
+          cudaMemcpy(&v, c->ws + c->lay.seq_tokens + (size_t)seq * 4, 4, cudaMemcpyDeviceToHost) !=
+              cudaSuccess)
+        return MD_ERR_CUDA;
+      *out = v;
+      return MD_OK;
+    }
     case MD_QUERY_PAGES: *out = c->n_pages[seq]; return MD_OK;
     case MD_QUERY_FREE_TOP: *out = c->m.free_top; return MD_OK;
     case MD_QUERY_STEP: *out = c->m.t; return MD_OK;
@@ -918,7 +1002,7 @@ MD_API md_status md_query(const md_ctx *c, int what, int seq, int64_t *out) {
 namespace {
 size_t host_blob_bytes(const md_ctx *c) {
   const size_t B = c->cfg.max_batch;
-  return sizeof(HostMirror) + sizeof(RegionTable) + B * (8 + 4 + 4 + 1);
+  return sizeof(HostMirror) + sizeof(RegionTable) + B * (8 + 4 + 4 + 1 + 4 + 4 + 1);
 }
 }  // namespace
 
@@ -959,6 +1043,12 @@ MD_API md_status md_save_state(md_ctx *c, void *dst_dev, void *host_blob) {
   memcpy(h, c->pinned_pages.data(), B * 4);
   h += B * 4;
   memcpy(h, c->tail_pinned.data(), B);
+  h += B;
+  memcpy(h, c->tail_fill.data(), B * 4);
+  h += B * 4;
+  memcpy(h, c->tail_region.data(), B * 4);
+  h += B * 4;
+  memcpy(h, c->tokens_exact.data(), B);
   return MD_OK;
 }
 
@@ -986,6 +1076,12 @@ MD_API md_status md_load_state(md_ctx *c, const void *src_dev, const void *host_
   memcpy(c->pinned_pages.data(), h, B * 4);
   h += B * 4;
   memcpy(c->tail_pinned.data(), h, B);
+  h += B;
+  memcpy(c->tail_fill.data(), h, B * 4);
+  h += B * 4;
+  memcpy(c->tail_region.data(), h, B * 4);
+  h += B * 4;
+  memcpy(c->tokens_exact.data(), h, B);
   return MD_OK;
 }
 

@@ -30,7 +30,8 @@ struct RegionTable {
 /* Byte offsets of every array inside the caller's workspace. */
 struct Layout {
   size_t pool, block_table, page_score, free_stack, region, a, t_ref, t_ins, window, ahat, prio, mass,
-      scratch, partials, counters, evict_list, staging_regions, staging_steps, status, calib, total;
+      scratch, partials, counters, evict_list, staging_regions, staging_steps, staging_slots, status,
+      calib, page_fill, seq_tokens, total;
   size_t slots, n_items;
   int scratch_tokens, chunk_stride;
 };
@@ -49,12 +50,16 @@ struct AppendParams {
   long long sb, sl, sh, si;              // element strides of the source (seq, layer, head, token)
   const uint8_t *regions_dev;            // per token (prefill) or null
   const int32_t *steps_dev;              // per token (prefill) or null
+  const int32_t *slots_dev;              // per token slot in the sequence (prefill) or null
+  uint8_t *page_fill;                    // [max_batch][P_max] tokens per page
+  int32_t *seq_tokens;                   // [max_batch] tokens per sequence
   int L, Hkv, ps, P_phys, P_max;         // L: layers written by this launch
   int l0;                                // first pool layer written
   int init_state;                        // 1: start token state, record new pages
   int lookup_only;                       // 1: pages already in the block table
   int n_seqs, n_per_seq, seq0, insert_step;
-  int tok0[MD_MAX_BATCH];                // cached tokens before this append
+  int tok0[MD_MAX_BATCH];                // slot of the first token (slots_dev == null)
+  int pages_before[MD_MAX_BATCH];        // pages of the sequence before this append
   int pop_base[MD_MAX_BATCH];            // free-stack index of the first page taken
   uint8_t regions_param[MD_MAX_BATCH];   // decode: region of each new token
 };
@@ -65,6 +70,8 @@ struct AttnParams {
   const uint16_t *q;
   uint16_t *out;
   const int32_t *block_table;
+  const uint8_t *page_fill;  // [max_batch][P_max] tokens per page, or null: pages are
+                             // full up to n_tokens
   float *mass;         // [L*Hkv][slots]
   float *scratch;      // [grid][2][scratch_tokens][8]
   float *partials;     // [items][chunk_stride][PARTIAL_FLOATS]
@@ -98,6 +105,8 @@ struct ScoreParams {
   const int32_t *t_ins;
   const uint8_t *region;
   const int32_t *block_table;
+  const uint8_t *page_fill;        // [max_batch][P_max] tokens per page
+  const int32_t *seq_tokens;       // [max_batch] |K_t| per sequence
   unsigned long long *calib_sum;   // [8][CALIB_BUCKETS] observed mass, fixed point 2^-32
   unsigned int *calib_cnt;         // [8][CALIB_BUCKETS] observations
   int calib_on;
@@ -125,6 +134,8 @@ struct SelectParams {
   int32_t *free_stack;
   int32_t *evict_list;    // [max_batch][P_max] internal
   int32_t *user_evicted;  // optional [n_seqs][P_max]
+  uint8_t *page_fill;     // [max_batch][P_max], compacted with the block table
+  int32_t *seq_tokens;    // [max_batch], less the evicted pages' tokens
   int *status;
   int P_max, n_seqs, top;
   int n_pages[MD_MAX_BATCH];

@@ -58,9 +58,9 @@ __global__ void append_kernel(const __grid_constant__ AppendParams p) {
     const int i = (int)(r % p.n_per_seq);
     const int j = (int)(r / p.n_per_seq);
     const int seq = p.seq0 + j;
-    const int tok = p.tok0[j] + i;
+    const int tok = p.slots_dev ? p.slots_dev[i] : p.tok0[j] + i;   // slot in the sequence
     const int pg = tok / p.ps, off = tok - pg * p.ps;
-    const int pages_before = p.lookup_only ? 0x7fffffff : (p.tok0[j] + p.ps - 1) / p.ps;
+    const int pages_before = p.lookup_only ? 0x7fffffff : p.pages_before[j];
     int phys;
     if (pg < pages_before)
       phys = p.block_table[(size_t)seq * p.P_max + pg];
@@ -84,6 +84,10 @@ __global__ void append_kernel(const __grid_constant__ AppendParams p) {
       p.ahat[slot] = 0.f;
       p.prio[slot] = 0.f;
       if (off == 0 && pg >= pages_before) p.block_table[(size_t)seq * p.P_max + pg] = phys;
+      /* the last token this append puts on a page sets the page's fill */
+      const int next = (i + 1 < p.n_per_seq) ? (p.slots_dev ? p.slots_dev[i + 1] : tok + 1) : -1;
+      if (next < 0 || next / p.ps != pg) p.page_fill[(size_t)seq * p.P_max + pg] = (uint8_t)(off + 1);
+      if (i == 0) p.seq_tokens[seq] += p.n_per_seq;
     }
   }
 }
@@ -170,7 +174,8 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
       b = find_seq(p.page_start, p.n_seqs, gp);
       pg = gp - p.page_start[b];
       P = p.n_pages[b];
-      valid = pg * PS + off < p.n_tokens[b];
+      valid = p.page_fill ? off < p.page_fill[(size_t)b * p.P_max + pg]
+                          : pg * PS + off < p.n_tokens[b];
       slot = (size_t)p.block_table[(size_t)b * p.P_max + pg] * PS + off;
     }
     float s = 0.f;
@@ -187,7 +192,8 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
           if (p.mass_pending) w += sum_rows(p.mass, p.slots, p.rows, slot);
           const float abar = __fdiv_rn(w, p.norm);                    // Sec. III-C
           a = p.rho * a + p.gamma * abar;                             // Eq. 2
-          const float tau = __fdiv_rn(p.tau_scale, (float)p.n_tokens[b]);
+          const int ntok = p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b];
+          const float tau = __fdiv_rn(p.tau_scale, (float)ntok);
           if (abar >= tau) tr = p.t;                                  // Eq. 3
           p.window[slot] = 0.f;
           p.ahat[slot] = abar;
@@ -207,7 +213,10 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
         switch (p.score_mode) {
           case 0: s = p.reg.base[reg] * d + p.alpha * a; break;       // Eq. 4
           case 1: s = (p.reg.base[reg] + p.alpha * a) * d; break;
-          case 2: s = p.reg.base[reg] * d + p.alpha * a * (float)p.n_tokens[b]; break;
+          case 2:
+            s = p.reg.base[reg] * d +
+                p.alpha * a * (float)(p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b]);
+            break;
           case 3: s = (float)p.t_ins[slot]; break;                     // recency
           default: s = random_draw(p.random_seed, p.t, slot); break;   // random
         }
@@ -299,10 +308,11 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
   extern __shared__ uint32_t sm[];
   uint32_t *keys = sm;                               // [P_max]
   int32_t *phys = (int32_t *)(sm + p.P_max);         // [P_max]
+  uint8_t *fills = (uint8_t *)(sm + 2 * (size_t)p.P_max);   // [P_max]
   __shared__ int hist[256];
   __shared__ int warp_sums[32];
   __shared__ uint32_t s_prefix;
-  __shared__ int s_k, s_bad;
+  __shared__ int s_k, s_bad, s_gone;
 
   const int b = blockIdx.x;
   const int P = p.n_pages[b];
@@ -315,12 +325,14 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
     return;
   }
   const float *sc = p.page_score + (size_t)b * p.P_max;
+  uint8_t *frow = p.page_fill + (size_t)b * p.P_max;
   for (int i = threadIdx.x; i < P; i += blockDim.x) {
     const float S = sc[i];
     keys[i] = (S == INFINITY) ? KEY_PINNED : order_key(S);
     phys[i] = row[i];
+    fills[i] = frow[i];
   }
-  if (threadIdx.x == 0) { s_prefix = 0u; s_k = e; s_bad = 0; }
+  if (threadIdx.x == 0) { s_prefix = 0u; s_k = e; s_bad = 0; s_gone = 0; }
   __syncthreads();
 
   /* radix select of the e-th smallest evictable key, most significant digit first */
@@ -356,7 +368,7 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
 
   /* evict: key < T, or key == T among the first take_eq in logical order;
    * compact kept pages in order; list the evicted ones in logical order */
-  int carry_eq = 0, carry_ev = 0;
+  int carry_eq = 0, carry_ev = 0, gone = 0;
   const int base_push = p.top + p.push_off[b];
   for (int t0 = 0; t0 < P; t0 += blockDim.x) {
     const int i = t0 + threadIdx.x;
@@ -374,22 +386,29 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
         p.evict_list[(size_t)b * p.P_max + idx_ev] = id;
         p.free_stack[base_push + idx_ev] = id;
         if (uout) uout[idx_ev] = id;
+        gone += fills[i];
       } else {
         row[i - idx_ev] = id;
+        frow[i - idx_ev] = fills[i];
       }
     }
     carry_eq += tot_eq;
     carry_ev += tot_ev;
   }
+  if (gone) atomicAdd(&s_gone, gone);
   __syncthreads();
-  for (int i = P - e + threadIdx.x; i < P; i += blockDim.x) row[i] = -1;
+  if (threadIdx.x == 0) p.seq_tokens[b] -= s_gone;
+  for (int i = P - e + threadIdx.x; i < P; i += blockDim.x) {
+    row[i] = -1;
+    frow[i] = 0;
+  }
   if (uout)
     for (int i = e + threadIdx.x; i < p.P_max; i += blockDim.x) uout[i] = -1;
 }
 
 cudaError_t launch_select(const SelectParams &p, cudaStream_t s) {
   if (p.n_seqs == 0) return cudaSuccess;
-  const size_t smem = (size_t)p.P_max * 8;
+  const size_t smem = (size_t)p.P_max * 9;
   cudaError_t err = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
   if (err != cudaSuccess) return err;

@@ -57,9 +57,14 @@ class Lockstep:
         kw = dict(rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
                   score_mode=w.score_mode, page_reduce=w.page_reduce,
                   random_seed=w.extra.get("random_seed", 0))
-        self.gpu = md.Cache(w.L, w.Hq, w.Hkv, w.page_size, B, self.P_max, self.P_phys, **kw)
+        aligned = bool(w.extra.get("region_aligned", False))
+        if aligned:    # a fresh page per region span can take up to one extra page per span
+            self.P_max += w.extra.get("extra_pages", 64)
+            self.P_phys += B * w.extra.get("extra_pages", 64)
+        self.gpu = md.Cache(w.L, w.Hq, w.Hkv, w.page_size, B, self.P_max, self.P_phys,
+                            region_aligned_pages=int(aligned), **kw)
         self.orc = om.Oracle(om.OracleConfig(w.L, w.Hq, w.Hkv, w.D, w.page_size, B, self.P_max,
-                                             self.P_phys, **kw))
+                                             self.P_phys, region_aligned=aligned, **kw))
         for r in range(7):
             self.gpu.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
             self.orc.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
@@ -118,6 +123,9 @@ class Lockstep:
         g = self.gpu
         o = self.orc
         pre_block = [list(o.block[b]) for b in range(B)]
+        pre_fill = [list(o.fill[b]) for b in range(B)]
+        pre_slots = [o.slots(b) for b in range(B)]
+        pre_pages = [o.page_of_token(b) for b in range(B)]
         observed = o.window_steps > 0
         st_g, n_g = g.evict(budgets)
         st_o, n_o, ids_o, logical_o = o.evict(B, budgets)
@@ -137,8 +145,8 @@ class Lockstep:
         fix_blocks = False
         for b in range(B):
             # the slots observed this step are those of the pre-eviction block table
-            n_pre = o.n_tokens[b] + len(logical_o[b]) * ps
-            sl = np.array([pre_block[b][i // ps] * ps + i % ps for i in range(n_pre)], np.int64)
+            sl = pre_slots[b]
+            n_pre = len(sl)
             if observed:
                 e = rel_err(ahat[sl], o.abar[sl])
                 self.max_err["ahat"] = max(self.max_err["ahat"], e)
@@ -165,8 +173,7 @@ class Lockstep:
             S_o = o.page_S[b]
             S_g = pscore[b, :P_pre].astype(np.float64)
             page_flip = np.zeros(P_pre, bool)
-            for i in np.nonzero(flipped)[0]:
-                page_flip[i // ps] = True
+            page_flip[pre_pages[b][np.nonzero(flipped)[0]]] = True
             e = rel_err(S_g[~page_flip], S_o[~page_flip])
             self.max_err["page"] = max(self.max_err["page"], e)
             assert e <= TOL_REL, f"page score rel err {e} (seq {b})"
@@ -207,13 +214,20 @@ class Lockstep:
         o = self.orc
         B = self.w.B
         bt = bt.copy()
+        fill = self.gpu.get_state(md.MD_STATE_PAGE_FILL).cpu().numpy()
+        ntok = self.gpu.get_state(md.MD_STATE_SEQ_TOKENS).cpu().numpy()
         for b in range(B):
             bt[b, :] = -1
             bt[b, :len(o.block[b])] = o.block[b]
+            fill[b, :] = 0
+            fill[b, :len(o.fill[b])] = o.fill[b]
+            ntok[b] = o.n_tokens[b]
         free = free.copy()
         free[:len(o.free)] = o.free
         self.gpu.set_state(md.MD_STATE_BLOCK_TABLE, torch.from_numpy(bt).cuda())
         self.gpu.set_state(md.MD_STATE_FREE, torch.from_numpy(free).cuda())
+        self.gpu.set_state(md.MD_STATE_PAGE_FILL, torch.from_numpy(fill).cuda())
+        self.gpu.set_state(md.MD_STATE_SEQ_TOKENS, torch.from_numpy(ntok).cuda())
 
     def check_calibration(self):
         """Histogram counts bit-exact, mass sums within the Abar tolerance (plus
@@ -235,9 +249,12 @@ class Lockstep:
         bt = self.gpu.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
         free = self.gpu.get_state(md.MD_STATE_FREE).cpu().numpy()
         o = self.orc
+        fill = self.gpu.get_state(md.MD_STATE_PAGE_FILL).cpu().numpy()
+        ntok = self.gpu.get_state(md.MD_STATE_SEQ_TOKENS).cpu().numpy()
         for b in range(self.w.B):
             assert list(bt[b, :len(o.block[b])]) == o.block[b]
-            assert self.gpu.query(md.MD_QUERY_TOKENS, b) == o.n_tokens[b]
+            assert list(fill[b, :len(o.fill[b])]) == o.fill[b]
+            assert self.gpu.query(md.MD_QUERY_TOKENS, b) == o.n_tokens[b] == ntok[b]
         assert self.gpu.query(md.MD_QUERY_FREE_TOP) == len(o.free)
         assert list(free[:len(o.free)]) == o.free
 

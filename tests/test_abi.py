@@ -41,7 +41,7 @@ def _cfg(**kw):
     c = dict(num_layers=2, num_q_heads=16, num_kv_heads=2, head_dim=128, page_size=16,
              max_batch=4, max_pages_per_seq=64, num_phys_pages=256, rho=0.9, gamma=0.1,
              tau_scale=2.0, attn_weight=1.0, score_mode=0, page_reduce=0, keep_token_prio=1,
-             workspace=None, workspace_bytes=0, stream=None, random_seed=0)
+             workspace=None, workspace_bytes=0, stream=None, random_seed=0, region_aligned_pages=0)
     c.update(kw)
     return md.md_config(*[c[f] for f, _ in md.md_config._fields_])
 

@@ -101,6 +101,27 @@ def test_policy_variants(mode):
         Lockstep(h2o).run().check_layout()
 
 
+def test_region_aligned_pages():
+    """Region-aligned allocation (a fresh page at each region boundary): no
+    page straddles two regions, pages are partly filled, every stage masks by
+    page fill, and eviction removes exactly the evicted pages' tokens."""
+    w = synth.custom_workload("aligned", L=2, Hq=16, Hkv=2, page_size=16, lengths=[700, 1900],
+                              budget_frac=0.5, steps=20, seed=18, structured=True)
+    w.extra["region_aligned"] = True
+    ls = Lockstep(w)
+    ls.prefill()
+    ls.check_layout()
+    assert any(f < 16 for f in ls.orc.fill[0][:-1])          # partial interior pages
+    for s in range(w.steps):
+        ls.decode(regions=[[6, 2][s % 2]] * w.B)            # alternating regions: page per switch
+        ls.observe()
+    ls.check_layout()
+    w2 = synth.custom_workload("aligned32", L=1, Hq=12, Hkv=2, page_size=32, lengths=[1500],
+                               budget_frac=0.4, steps=8, seed=19, window_k=2)
+    w2.extra["region_aligned"] = True
+    Lockstep(w2, layerwise=True).run().check_layout()
+
+
 def test_pins_over_budget_warns():
     """Pinned pages alone exceed the budget: every evictable page goes, the
     warning comes back, pinned pages stay."""

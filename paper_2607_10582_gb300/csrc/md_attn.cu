@@ -19,11 +19,14 @@
  *
  * Exact mass without re-reading K: a token's mass is sum_h exp(s_hi - m_h)/Z_h
  * with the item's global (m_h, Z_h).  A unit publishes its partial (m, Z, O)
- * and bumps the item's arrival counter; one unit later (so nothing waits on
- * the critical path) the CTA waits, bounded by %globaltimer, for all chunks of
- * the earlier item, combines the partials (its slice of the output O) and
- * turns its stored scores into masses, one fp32 row per (layer, KV head)
- * indexed by physical slot.  All waits are bounded; on expiry the kernel
+ * and bumps the item's arrival counter.  The last warp of the CTA, the
+ * finisher, then takes the unit over while the consumers stream the next
+ * one: it waits, bounded by %globaltimer, for all chunks of the item,
+ * combines the partials (its slice of the output O) and turns the stored
+ * scores into masses, one fp32 row per (layer, KV head) indexed by physical
+ * slot.  Raw scores live in two slots per CTA; the consumers reuse a slot only
+ * after the finisher has released it (mbarrier hand-off both ways), so the
+ * finish never stalls the copy stream.  All waits are bounded; on expiry the kernel
  * records MD_ERR_DEVICE_TIMEOUT, raises an abort flag every CTA polls, drains
  * its in-flight copies and returns.  No float atomics: results are
  * bit-identical run to run. */
@@ -43,13 +46,15 @@ struct AttnShape {
   static constexpr int R = (PS == 16) ? 8 : 4;       // ring stages (64 KiB per CTA)
   static constexpr int RING_BYTES = R * STAGE_BYTES;
   static constexpr int CTAS_PER_SM = 2;
-  static constexpr int THREADS = 32 * (NCW + 1);
+  static constexpr int THREADS = 32 * (NCW + 2);     // producer, NCW consumers, finisher
   static constexpr int Q_BYTES = GP * D * 2;         // one unit's query heads
   static constexpr int MAX_UNIT_PAGES = MD_MAX_CHUNK_TOKENS / PS;
   static constexpr int MERGE_FLOATS = NCW * (24 + GP * D);
   static constexpr int FIN_FLOATS = 16 + 3 * MD_MAX_CHUNKS * GP;
-  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * Q_BYTES + (2 * R + 4) * 8 +
-                                 4 * MERGE_FLOATS + 4 * FIN_FLOATS + 8 * MAX_UNIT_PAGES + 4 * R + 64;
+  static constexpr int OBUF_FLOATS = GP * D + MD_MAX_CHUNKS;   // C slices of ceil(G*D/C)
+  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * Q_BYTES + (2 * R + 8) * 8 +
+                                 4 * MERGE_FLOATS + 4 * FIN_FLOATS + 8 * MAX_UNIT_PAGES +
+                                 4 * OBUF_FLOATS + 4 * R + 64;
 };
 
 struct Unit {
@@ -108,6 +113,208 @@ __device__ __forceinline__ uint32_t swz(uint32_t stage, int row, int d) {
   return stage + half * (2 * PS * 128) + row * 128 + ((chunk ^ (row & 7)) << 4);
 }
 
+/* Shared memory of the end-of-unit pass. */
+struct FinSmem {
+  float *fin;     // [16]: head max, then 1/Z
+  float *pm, *pl; // [MD_MAX_CHUNKS][8] partial maxima and sums
+  float *fac;     // [MD_MAX_CHUNKS][8] combine factors
+  float *obuf;    // staged partial O slices
+  int *sphys;     // [unit pages] physical page ids
+  int *sfill;     // [unit pages] tokens per page (region-aligned pages)
+  int *okflag;    // the bounded wait's outcome, for every thread
+};
+
+template <int NT>
+__device__ __forceinline__ void fin_sync() {
+  if (NT == 32) __syncwarp();
+  else named_barrier(1, NT);
+}
+
+/* The end of a unit: wait (bounded) for all C chunks of its (sequence, layer,
+ * KV head) item, combine their partials (m, Z, O) into this chunk's slice of
+ * the output O and the item's per-head (max, 1/Z), turn the unit's stored
+ * scores into token masses sum_h exp2(s_hi - max_h) / Z_h (Sec. III-C), then
+ * count the chunk as finished.  Run by NT threads, tid < NT: the finisher
+ * warp, or all consumer warps for a CTA's last unit.  Returns false, the same
+ * for every thread, on abort or timeout.  Loads are issued in batches before
+ * the dependent stores, so a pass costs a few L2 round trips. */
+template <int PS, bool ALIGNED, int NT, int OBUF_FLOATS>
+__device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv, int slot, int tid,
+                                            const FinSmem &f) {
+  const float NEG_INF = -INFINITY;
+  const int G = p.G;
+  const int npg = pv.p1 - pv.p0;
+  const int C = pv.C;
+  /* the unit's page ids (no wait needed) */
+  const int32_t *bt = p.block_table + (size_t)pv.b * p.P_max;
+  for (int q0 = 0; q0 < npg; q0 += NT * 4) {
+    int ph[4], fl[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int q = q0 + r * NT + tid;
+      ph[r] = fl[r] = 0;
+      if (q < npg) {
+        ph[r] = bt[pv.p0 + q];
+        if (ALIGNED) fl[r] = p.page_fill[(size_t)pv.b * p.P_max + pv.p0 + q];
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int q = q0 + r * NT + tid;
+      if (q < npg) {
+        f.sphys[q] = ph[r];
+        if (ALIGNED) f.sfill[q] = fl[r];
+      }
+    }
+  }
+  /* all chunks of the item published */
+  if (tid == 0) {
+    int okw = 1;
+    const int target = C + p.extra_arrivals;
+    if (ld_acquire_gpu(&p.counters[pv.X]) < target) {
+      const long long t0 = globaltimer();
+      while (ld_acquire_gpu(&p.counters[pv.X]) < target) {
+        if (ld_volatile(&p.status[ST_ABORT])) { okw = 0; break; }
+        if (globaltimer() - t0 > p.spin_limit_ns) {
+          raise_status(p, MD_ERR_DEVICE_TIMEOUT, 3);
+          okw = 0;
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    *f.okflag = okw;
+  }
+  fin_sync<NT>();
+  if (!*f.okflag) return false;
+  const float *base = p.partials + (size_t)pv.X * p.chunk_stride * PARTIAL_FLOATS;
+  for (int i0 = 0; i0 < C * GP; i0 += NT * 8) {
+    float vm[8], vl[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const int idx = i0 + r * NT + tid;
+      vm[r] = vl[r] = 0.f;
+      if (idx < C * GP) {
+        const float *pj = base + (size_t)(idx >> 3) * PARTIAL_FLOATS;
+        vm[r] = __ldcg(pj + (idx & 7));
+        vl[r] = __ldcg(pj + 8 + (idx & 7));
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const int idx = i0 + r * NT + tid;
+      if (idx < C * GP) {
+        f.pm[idx] = vm[r];
+        f.pl[idx] = vl[r];
+      }
+    }
+  }
+  fin_sync<NT>();
+  if (tid < 32) {
+    /* per head: global max and normaliser over the C chunks */
+    const int h = tid & 7, part = tid >> 3;
+    float M = NEG_INF;
+    for (int j = part; j < C; j += 4) M = fmaxf(M, f.pm[j * GP + h]);
+    M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 8));
+    M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 16));
+    const float Mr = (M == NEG_INF) ? 0.f : M;
+    float Z = 0.f;
+    for (int j = part; j < C; j += 4) Z += exp2f(f.pm[j * GP + h] - Mr) * f.pl[j * GP + h];
+    Z += __shfl_xor_sync(0xffffffffu, Z, 8);
+    Z += __shfl_xor_sync(0xffffffffu, Z, 16);
+    if (part == 0) {
+      f.fin[h] = Mr;
+      f.fin[8 + h] = Z > 0.f ? 1.f / Z : 0.f;
+    }
+  }
+  fin_sync<NT>();
+  for (int idx = tid; idx < C * GP; idx += NT)
+    f.fac[idx] = exp2f(f.pm[idx] - f.fin[idx & 7]) * f.fin[8 + (idx & 7)];
+  /* this chunk's slice [lo, hi) of the item's output O[h][d] (h < G): the C
+   * partial slices are staged in shared memory with independent loads (one
+   * batch, all in flight), then each thread sums its elements' chunks in
+   * chunk order */
+  const int E = G * D;
+  const int lo = (int)(((long long)pv.j * E) / C);
+  const int hi = (int)(((long long)(pv.j + 1) * E) / C);
+  const int SE = hi - lo;
+  const int n_all = C * SE;   // <= E + C - 1 < OBUF_FLOATS
+  {
+    constexpr int NBO = (OBUF_FLOATS + NT - 1) / NT;
+    float v[NBO];
+#pragma unroll
+    for (int r = 0; r < NBO; ++r) {
+      const int n = r * NT + tid;
+      v[r] = 0.f;
+      if (n < n_all) {
+        const int j = n / SE;
+        v[r] = __ldcg(base + (size_t)j * PARTIAL_FLOATS + 16 + lo + (n - j * SE));
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < NBO; ++r) {
+      const int n = r * NT + tid;
+      if (n < n_all) f.obuf[n] = v[r];
+    }
+  }
+  fin_sync<NT>();
+  {
+    uint16_t *orow = p.out + (((size_t)pv.b * p.q_layers + (pv.l - p.l0)) * p.Hq + (size_t)pv.kvh * G) * D;
+    for (int e = lo + tid; e < hi; e += NT) {
+      const int h = e >> 7;
+      float acc = 0.f;
+      for (int j = 0; j < C; ++j) acc += f.fac[j * GP + h] * f.obuf[j * SE + (e - lo)];
+      __nv_bfloat16 bv = __float2bfloat16_rn(acc);
+      orow[e] = *(uint16_t *)&bv;
+    }
+  }
+  /* token masses of this chunk from its stored scores, eight tokens per
+   * thread in flight (a batch's loads are issued before any store) */
+  {
+    const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + slot) * p.scratch_tokens * GP;
+    const int ntok = npg * PS;
+    float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
+    float fm[GP], fz[GP];
+#pragma unroll
+    for (int h = 0; h < GP; ++h) {
+      fm[h] = f.fin[h];
+      fz[h] = (h < G) ? f.fin[8 + h] : 0.f;
+    }
+    /* contiguous pages: the valid tokens are a prefix of the unit; with
+     * region-aligned pages every page has its own fill */
+    const int nvalid = ALIGNED ? ntok : min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
+    constexpr int NB = 8;
+    for (int tk0 = 0; tk0 < nvalid; tk0 += NT * NB) {
+      float4 s0[NB], s1[NB];
+#pragma unroll
+      for (int r = 0; r < NB; ++r) {
+        const int tk = tk0 + r * NT + tid;
+        if (tk < nvalid) {
+          s0[r] = __ldcg((const float4 *)(scr + (size_t)tk * GP));
+          s1[r] = __ldcg((const float4 *)(scr + (size_t)tk * GP + 4));
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < NB; ++r) {
+        const int tk = tk0 + r * NT + tid;
+        if (tk >= nvalid) continue;
+        if (ALIGNED && (tk % PS) >= f.sfill[tk / PS]) continue;
+        float m = exp2f(s0[r].x - fm[0]) * fz[0] + exp2f(s0[r].y - fm[1]) * fz[1] +
+                  exp2f(s0[r].z - fm[2]) * fz[2] + exp2f(s0[r].w - fm[3]) * fz[3];
+        m += exp2f(s1[r].x - fm[4]) * fz[4] + exp2f(s1[r].y - fm[5]) * fz[5] +
+             exp2f(s1[r].z - fm[6]) * fz[6] + exp2f(s1[r].w - fm[7]) * fz[7];
+        mrow[(size_t)f.sphys[tk / PS] * PS + (tk % PS)] = m;
+      }
+    }
+  }
+  fin_sync<NT>();
+  if (tid == 0) {
+    const int old = atomicAdd(&p.counters[pv.X], 1);
+    if (old == 2 * C - 1) atomicExch(&p.counters[pv.X], 0);
+  }
+  return true;
+}
+
 /* ALIGNED: pages carry their own fill (region-aligned allocation); otherwise
  * every page but the last is full and the fills follow from n_tokens. */
 template <int PS, int NCW, bool ALIGNED>
@@ -123,7 +330,9 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   uint64_t *empty = full + S::R;
   uint64_t *qfull = empty + S::R;                       // [2]
   uint64_t *qempty = qfull + 2;                         // [2]
-  float *wm = (float *)(qempty + 2);          // [NCW][8] per-warp running max
+  uint64_t *cdone = qempty + 2;    // [2] score slot written, unit published
+  uint64_t *fdone = cdone + 2;     // [2] score slot read by the finisher
+  float *wm = (float *)(fdone + 2);           // [NCW][8] per-warp running max
   float *wl = wm + NCW * 8;                   // [NCW][8] per-warp running sum
   float *wf = wl + NCW * 8;                   // [NCW][8] per-warp merge factor
   float *wO = wf + NCW * 8;                   // [NCW][8][128] per-warp O^T
@@ -133,7 +342,8 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   float *fac = pl + MD_MAX_CHUNKS * GP;       // [MD_MAX_CHUNKS][8] combine factors
   int *sphys = (int *)(fac + MD_MAX_CHUNKS * GP);   // [MAX_UNIT_PAGES] page ids
   int *sfill = sphys + S::MAX_UNIT_PAGES;            // [MAX_UNIT_PAGES] tokens per page
-  int *fillbuf = sfill + S::MAX_UNIT_PAGES;          // [R] fill of the page in each stage
+  float *obuf = (float *)(sfill + S::MAX_UNIT_PAGES);   // [OBUF_FLOATS] staged O slices
+  int *fillbuf = (int *)(obuf + S::OBUF_FLOATS);         // [R] fill of the page in each stage
   int *flag = fillbuf + S::R;
 
   const int warp = threadIdx.x >> 5;
@@ -150,8 +360,10 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     for (int s = 0; s < 2; ++s) {
       mbar_init(smem_u32(&qfull[s]), 1);
       mbar_init(smem_u32(&qempty[s]), NCW);
+      mbar_init(smem_u32(&cdone[s]), 1);
+      mbar_init(smem_u32(&fdone[s]), 1);
     }
-    flag[0] = flag[1] = flag[2] = 0;
+    flag[0] = flag[1] = flag[2] = flag[3] = 0;
     fence_barrier_init();
   }
   __syncthreads();
@@ -218,6 +430,24 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     return;
   }
 
+  const FinSmem fs{fin, pm, pl, fac, obuf, sphys, sfill, &flag[2]};
+
+  if (warp == NCW + 1) {
+    /* ------------------------------------------------------- finisher ---- */
+    /* The end of every unit but the CTA's last, one warp, while the
+     * consumers stream the next unit; then the score slot is released. */
+    int k = 0;
+    for (int u = blockIdx.x; u < p.total_units; u += gridDim.x, ++k) {
+      if (u + (int)gridDim.x >= p.total_units) break;   // the consumers finish the last unit
+      const Unit pv = decode_unit(p, u);
+      const bool ok = wait_phase(smem_u32(&cdone[k & 1]), (k >> 1) & 1, p, 8, true);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      if (!finish_unit<PS, ALIGNED, 32, S::OBUF_FLOATS>(p, pv, k & 1, lane, fs)) break;
+      if (lane == 0) mbar_arrive(smem_u32(&fdone[k & 1]));   // slot and finish area free
+    }
+    return;
+  }
+
   /* ------------------------------------------------------- consumers ----- */
   const int cw = warp - 1;
   const int ct = threadIdx.x - 32;
@@ -228,126 +458,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   const float NEG_INF = -INFINITY;
 
   int i_base = 0, nunit = 0;
-  bool have_prev = false;
-  Unit prev{};
   bool aborted = false;   // this warp gave up a wait
-  bool stopped = false;   // all consumer warps leave the unit loop together
-
-  /* Deferred end of a unit: wait for the item's other chunks, combine the
-   * partials (this chunk's slice of O), turn the stored scores into masses. */
-  auto finish = [&](const Unit &pv, int pv_slot) -> bool {
-    if (ct == 0) {
-      const int target = pv.C + p.extra_arrivals;
-      int okw = 1;
-      if (ld_acquire_gpu(&p.counters[pv.X]) < target) {
-        const long long t0 = globaltimer();
-        while (ld_acquire_gpu(&p.counters[pv.X]) < target) {
-          if (ld_volatile(&p.status[ST_ABORT])) { okw = 0; break; }
-          if (globaltimer() - t0 > p.spin_limit_ns) {
-            raise_status(p, MD_ERR_DEVICE_TIMEOUT, 3);
-            okw = 0;
-            break;
-          }
-          __nanosleep(64);
-        }
-      }
-      flag[2] = okw ? 0 : 1;
-    }
-    named_barrier(1, NC);
-    if (flag[2]) return false;
-    const int C = pv.C;
-    const float *base = p.partials + (size_t)pv.X * p.chunk_stride * PARTIAL_FLOATS;
-    const int32_t *bt = p.block_table + (size_t)pv.b * p.P_max;
-    for (int idx = ct; idx < C * GP; idx += NC) {
-      const float *pj = base + (size_t)(idx >> 3) * PARTIAL_FLOATS;
-      pm[idx] = __ldcg(pj + (idx & 7));
-      pl[idx] = __ldcg(pj + 8 + (idx & 7));
-    }
-    for (int k = ct; k < pv.p1 - pv.p0; k += NC) {
-      sphys[k] = bt[pv.p0 + k];
-      if (ALIGNED) sfill[k] = p.page_fill[(size_t)pv.b * p.P_max + pv.p0 + k];
-    }
-    named_barrier(1, NC);
-    if (cw == 0) {
-      /* per head: global max and normaliser over the C chunks */
-      const int h = lane & 7, part = lane >> 3;
-      float M = NEG_INF;
-      for (int j = part; j < C; j += 4) M = fmaxf(M, pm[j * GP + h]);
-      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 8));
-      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 16));
-      const float Mr = (M == NEG_INF) ? 0.f : M;
-      float Z = 0.f;
-      for (int j = part; j < C; j += 4) Z += exp2f(pm[j * GP + h] - Mr) * pl[j * GP + h];
-      Z += __shfl_xor_sync(0xffffffffu, Z, 8);
-      Z += __shfl_xor_sync(0xffffffffu, Z, 16);
-      if (part == 0) {
-        fin[h] = Mr;
-        fin[8 + h] = Z > 0.f ? 1.f / Z : 0.f;
-      }
-    }
-    named_barrier(1, NC);
-    for (int idx = ct; idx < C * GP; idx += NC)
-      fac[idx] = exp2f(pm[idx] - fin[idx & 7]) * fin[8 + (idx & 7)];
-    named_barrier(1, NC);
-    /* this chunk's slice of the item's output O[h][d] (h < G): four threads
-     * per element, each summing a quarter of the chunks */
-    {
-      const int E = G * D;
-      const int lo = (int)(((long long)pv.j * E) / C);
-      const int hi = (int)(((long long)(pv.j + 1) * E) / C);
-      uint16_t *orow = p.out + (((size_t)pv.b * p.q_layers + (pv.l - p.l0)) * p.Hq + (size_t)pv.kvh * G) * D;
-      const int q4 = ct & 3;
-      for (int e0 = lo; e0 < hi; e0 += NC / 4) {
-        const int e = e0 + (ct >> 2);
-        float acc = 0.f;
-        if (e < hi) {
-          const int h = e >> 7;
-#pragma unroll 4
-          for (int j = q4; j < C; j += 4)
-            acc += fac[j * GP + h] * __ldcg(base + (size_t)j * PARTIAL_FLOATS + 16 + e);
-        }
-        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
-        if (q4 == 0 && e < hi) {
-          __nv_bfloat16 v = __float2bfloat16_rn(acc);
-          orow[e] = *(uint16_t *)&v;
-        }
-      }
-    }
-    /* token masses of this chunk from its stored scores */
-    {
-      const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + pv_slot) * p.scratch_tokens * GP;
-      const int ntok = (pv.p1 - pv.p0) * PS;
-      float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
-      float fm[GP], fz[GP];
-#pragma unroll
-      for (int h = 0; h < GP; ++h) {
-        fm[h] = fin[h];
-        fz[h] = (h < G) ? fin[8 + h] : 0.f;
-      }
-      /* contiguous pages: the valid tokens are a prefix of the unit; with
-       * region-aligned pages every page has its own fill */
-      const int nvalid = ALIGNED ? ntok : min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
-#pragma unroll 4
-      for (int tk = ct; tk < nvalid; tk += NC) {
-        if (ALIGNED && (tk % PS) >= sfill[tk / PS]) continue;
-        const float4 s0 = __ldcg((const float4 *)(scr + (size_t)tk * GP));
-        const float4 s1 = __ldcg((const float4 *)(scr + (size_t)tk * GP + 4));
-        float m = exp2f(s0.x - fm[0]) * fz[0] + exp2f(s0.y - fm[1]) * fz[1] +
-                  exp2f(s0.z - fm[2]) * fz[2] + exp2f(s0.w - fm[3]) * fz[3];
-        m += exp2f(s1.x - fm[4]) * fz[4] + exp2f(s1.y - fm[5]) * fz[5] +
-             exp2f(s1.z - fm[6]) * fz[6] + exp2f(s1.w - fm[7]) * fz[7];
-        mrow[(size_t)sphys[tk / PS] * PS + (tk % PS)] = m;
-      }
-    }
-    named_barrier(1, NC);
-    if (ct == 0) {
-      const int old = atomicAdd(&p.counters[pv.X], 1);
-      if (old == 2 * pv.C - 1) atomicExch(&p.counters[pv.X], 0);
-    }
-    return true;
-  };
-
   for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
     const Unit un = decode_unit(p, u);
     const int npg = un.p1 - un.p0;
@@ -375,6 +486,11 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&qempty[qs]));
     }
+    /* the score slot is free once the finisher is done with the unit that
+     * used it two units ago */
+    if (nunit >= 2 && !aborted &&
+        !wait_phase(smem_u32(&fdone[slot]), ((nunit >> 1) - 1) & 1, p, 9, true))
+      aborted = true;
     float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
     float o[8][4];
 #pragma unroll
@@ -484,7 +600,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     }
     if (aborted) flag[0] = 1;
     named_barrier(1, NC);
-    if (flag[0]) { stopped = true; break; }
+    if (flag[0]) break;
     float *part = p.partials + ((size_t)un.X * p.chunk_stride + un.j) * PARTIAL_FLOATS;
     if (ct < GP) {
       float M = NEG_INF;
@@ -514,15 +630,22 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       flag[1] = ld_volatile(&p.status[ST_ABORT]);
     }
     named_barrier(1, NC);
-    if (flag[1]) { stopped = true; break; }
-
-    if (have_prev && !finish(prev, (nunit - 1) & 1)) { stopped = true; break; }
-    prev = un;
-    have_prev = true;
+    if (flag[1]) break;
+    if (u + (int)gridDim.x >= p.total_units) {
+      /* the CTA's last unit: nothing is left to overlap with, so all consumer
+       * warps finish it, once the finisher has released the finish area */
+      if (ct == 0)
+        flag[3] = (nunit >= 1 && !wait_phase(smem_u32(&fdone[(nunit - 1) & 1]),
+                                              ((nunit - 1) >> 1) & 1, p, 9, true)) ? 1 : 0;
+      named_barrier(1, NC);
+      if (flag[3]) break;
+      finish_unit<PS, ALIGNED, NCW * 32, S::OBUF_FLOATS>(p, un, slot, ct, fs);
+      break;
+    }
+    if (ct == 0) mbar_arrive(smem_u32(&cdone[slot]));   // hand the unit to the finisher
     i_base += npg;
     ++nunit;
   }
-  if (!stopped && have_prev) finish(prev, (nunit - 1) & 1);
 }
 
 template <int PS, int NCW, bool AL>

@@ -269,8 +269,9 @@ md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_p
  *                             the kernel then reports MD_ERR_DEVICE_TIMEOUT)
  *   MD_DEBUG_GRID_LIMIT       cap on the attention kernel's persistent CTAs
  *                             (0 = all that fit on the device)
- *   MD_DEBUG_UNIT_OVERHEAD    per-unit cost, in pages, that the attention work
- *                             planner adds to each chunk (default 8)
+ *   MD_DEBUG_UNIT_OVERHEAD    per-unit cost, in KiB of K/V streamed, that the
+ *                             attention work planner adds to each chunk
+ *                             (default 112; 0..65536)
  *   MD_DEBUG_FORCE_CHUNKS     chunks per (sequence, layer, KV head) item
  *                             (0 = planned; otherwise clamped to the limits) */
 enum {

@@ -623,9 +623,11 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       for (int w = 0; w < NCW; ++w) acc += wf[w * 8 + h] * wO[(size_t)w * GP * D + e];
       part[16 + e] = acc;
     }
-    __threadfence();
+    /* release: the barrier orders every thread's partial (and score) writes
+     * before thread 0, whose gpu-scope fence is cumulative over them */
     named_barrier(1, NC);
     if (ct == 0) {
+      __threadfence();
       atomicAdd(&p.counters[un.X], 1);
       flag[1] = ld_volatile(&p.status[ST_ABORT]);
     }

@@ -64,8 +64,13 @@ struct md_ctx {
   long long spin_limit_ns = 2000000000LL;
   int extra_arrivals = 0;
   int grid_cap = 0;          // 0: every CTA that fits
-  int unit_overhead = 4;     // planner: per-unit cost in pages
+  int unit_overhead_kib = 112;   // planner: per-unit cost, as KiB of K/V streamed
   int force_chunks = 0;      // planner: 0 = choose
+  /* the planner's last choice of pages per chunk, reused while its inputs
+   * (batch, layers, knobs, pages per sequence) repeat */
+  std::vector<int> plan_pages;
+  int plan_batch = -1, plan_layers = -1, plan_T = 0;
+  int plan_knobs[4] = {-1, -1, -1, -1};
   bool calib_on = false;     // calibration histogram being gathered
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
@@ -243,10 +248,16 @@ md_status launch_fold(md_ctx *c) {
   return MD_OK;
 }
 
-/* Split every (sequence, layer, KV head) item's pages into chunks so that the
- * persistent grid gets balanced rounds: minimise rounds x (largest chunk +
- * a per-unit overhead), with at most MD_MAX_CHUNK_TOKENS tokens per chunk. */
-void plan_attention(const md_ctx *c, int batch, int layers, AttnParams &ap, int *grid) {
+/* Split every (sequence, layer, KV head) item's pages into chunks for the
+ * persistent grid, which takes units round-robin (unit u on CTA u mod G).
+ * Each candidate split is costed by its exact makespan under that schedule:
+ * a sequence's units are one contiguous run of unit ids, so every CTA gets
+ * floor(n_b / G) of them plus one more on a cyclic CTA interval, and a
+ * difference array gives all CTA loads in O(batch + G).  A unit costs its
+ * pages plus a fixed per-unit overhead (Q load, merge, publish, ramp),
+ * expressed as K/V bytes streamed.  At most MD_MAX_CHUNK_TOKENS tokens per
+ * chunk; the live raw-score scratch must stay inside L2. */
+void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid) {
   const int ps = c->cfg.page_size;
   const int items = layers * c->cfg.num_kv_heads;
   int Pmax = 1;
@@ -255,38 +266,79 @@ void plan_attention(const md_ctx *c, int batch, int layers, AttnParams &ap, int 
   const int cmax = c->lay.chunk_stride;
   const long long glim =
       c->grid_cap > 0 ? std::min<long long>(c->grid_cap, c->grid_limit) : c->grid_limit;
+  const double page_kib = ps * 512.0 / 1024.0;   // K+V of one (layer, KV head) page
+  const double ov = c->unit_overhead_kib / page_kib;
+  const int knobs[4] = {(int)glim, c->unit_overhead_kib, c->force_chunks, c->lay.scratch_tokens};
+  bool same = c->plan_batch == batch && c->plan_layers == layers &&
+              std::equal(knobs, knobs + 4, c->plan_knobs);
+  for (int b = 0; same && b < batch; ++b) same = c->plan_pages[b] == c->n_pages[b];
   double best = 1e300;
-  int bestT = 0;
+  int bestT = same ? c->plan_T : 0;
+  double diff[MAX_GRID + 1];
   /* Every CTA keeps the raw scores of two units in L2 (evict_last) until the
-   * unit after next; keep that set well inside L2 or its lines spill. */
-  const double l2_budget = 56.0 * (1 << 20);
+   * finisher has read them; keep that set well inside L2 or its lines spill. */
+  const double l2_budget = 46.0 * (1 << 20);
   for (int pass = 0; pass < 2 && bestT == 0; ++pass)
-  for (int C = 1; C <= cmax; ++C) {
+  for (int C = 1, Tprev = 0; C <= cmax; ++C) {
     const int T = (Pmax + C - 1) / C;
-    if (T > max_chunk_pages) continue;
-    if (pass == 0 && (double)glim * 2 * T * ps * GP * 4 > l2_budget) continue;
     if (c->force_chunks > 0) {
       const int need = (Pmax + max_chunk_pages - 1) / max_chunk_pages;
       if (C != std::min(cmax, std::max(c->force_chunks, need))) continue;
+    } else {
+      if (T == Tprev) continue;   // the same split as the previous candidate
+      Tprev = T;
     }
+    if (T > max_chunk_pages) continue;
+    if (pass == 0 && (double)glim * 2 * T * ps * GP * 4 > l2_budget) continue;
     long long U = 0;
-    int maxpg = 0;
+    for (int b = 0; b < batch; ++b) {
+      const int P = c->n_pages[b];
+      if (P > 0) U += (long long)items * std::min(std::min((P + T - 1) / T, cmax), P);
+    }
+    if (U == 0) continue;
+    const int G = (int)std::max(1LL, std::min<long long>(U, glim));
+    for (int g = 0; g <= G; ++g) diff[g] = 0.0;
+    double base = 0.0;
+    long long start = 0;
     for (int b = 0; b < batch; ++b) {
       const int P = c->n_pages[b];
       if (P == 0) continue;
-      int ch = std::min(std::min((P + T - 1) / T, cmax), P);
-      U += (long long)items * ch;
-      maxpg = std::max(maxpg, (P + ch - 1) / ch);
+      const int ch = std::min(std::min((P + T - 1) / T, cmax), P);
+      const long long n = (long long)items * ch;
+      const double sz = (double)P / ch + ov;
+      base += (double)(n / G) * sz;
+      const int r = (int)(n % G), s0 = (int)(start % G);
+      if (r > 0) {
+        diff[s0] += sz;
+        if (s0 + r <= G) {
+          diff[s0 + r] -= sz;
+        } else {
+          diff[G] -= sz;
+          diff[0] += sz;
+          diff[s0 + r - G] -= sz;
+        }
+      }
+      start += n;
     }
-    const long long G = std::max(1LL, std::min<long long>(U, glim));
-    const double rounds = (double)((U + G - 1) / G);
-    const double cost = rounds * (maxpg + (double)c->unit_overhead);
+    double run = 0.0, peak = 0.0;
+    for (int g = 0; g < G; ++g) {
+      run += diff[g];
+      peak = std::max(peak, run);
+    }
+    const double cost = base + peak;
     if (cost < best - 1e-9) {
       best = cost;
       bestT = T;
     }
   }
   if (bestT == 0) bestT = max_chunk_pages;
+  if (!same) {
+    c->plan_batch = batch;
+    c->plan_layers = layers;
+    std::copy(knobs, knobs + 4, c->plan_knobs);
+    c->plan_pages.assign(c->n_pages.begin(), c->n_pages.begin() + batch);
+    c->plan_T = bestT;
+  }
   long long U = 0;
   for (int b = 0; b < batch; ++b) {
     const int P = c->n_pages[b];
@@ -1136,8 +1188,8 @@ MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
     return MD_OK;
   }
   if (key == MD_DEBUG_UNIT_OVERHEAD) {
-    if (value < 0 || value > 4096) return fail(c, MD_ERR_INVALID_ARG, "unit overhead out of range");
-    c->unit_overhead = (int)value;
+    if (value < 0 || value > 65536) return fail(c, MD_ERR_INVALID_ARG, "unit overhead out of range");
+    c->unit_overhead_kib = (int)value;
     return MD_OK;
   }
   if (key == MD_DEBUG_FORCE_CHUNKS) {

@@ -10,7 +10,10 @@
  * Per CTA: warp 0 is the producer.  One elected lane issues, per page, two
  * TMA tile loads (cp.async.bulk.tensor, 128-byte swizzle, L2 evict_first) of
  * the page's K and V rows into a ring of shared-memory stages with mbarrier
- * completion.  Warps 1..NCW consume pages round-robin:
+ * completion.  Warps 1..NCW consume pages round-robin by the CTA-wide page
+ * index i (warp i % NCW, stage i % R), so each warp owns R / NCW stages: the
+ * warps may run up to a unit apart and no wait is ever more than one phase
+ * ahead:
  *   S^T[16 tokens x 8 heads] = K[16 x 128] . Q^T    (mma.sync m16n8k16 bf16)
  *   online softmax per head (exp2 domain), raw scores kept in scratch
  *   O^T[128 x 8] += V^T[128 x 16] . P^T             (P^T via movmatrix.trans)
@@ -44,6 +47,7 @@ struct AttnShape {
   static constexpr int HALF_BYTES = 2 * PS * 128;    // 64 columns of K and V rows
   static constexpr int STAGE_BYTES = 2 * HALF_BYTES; // one page of one (layer, KV head)
   static constexpr int R = (PS == 16) ? 8 : 4;       // ring stages (64 KiB per CTA)
+  static_assert(R % NCW == 0, "every consumer warp owns R / NCW stages");
   static constexpr int RING_BYTES = R * STAGE_BYTES;
   static constexpr int CTAS_PER_SM = 2;
   static constexpr int THREADS = 32 * (NCW + 2);     // producer, NCW consumers, finisher
@@ -52,7 +56,7 @@ struct AttnShape {
   static constexpr int MERGE_FLOATS = NCW * (24 + GP * D);
   static constexpr int FIN_FLOATS = 16 + 3 * MD_MAX_CHUNKS * GP;
   static constexpr int OBUF_FLOATS = GP * D + MD_MAX_CHUNKS;   // C slices of ceil(G*D/C)
-  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * Q_BYTES + (2 * R + 8) * 8 +
+  static constexpr size_t SMEM = 1024 + RING_BYTES + 2 * Q_BYTES + (2 * R + 10) * 8 +
                                  4 * MERGE_FLOATS + 4 * FIN_FLOATS + 8 * MAX_UNIT_PAGES +
                                  4 * OBUF_FLOATS + 4 * R + 64;
 };
@@ -130,22 +134,12 @@ __device__ __forceinline__ void fin_sync() {
   else named_barrier(1, NT);
 }
 
-/* The end of a unit: wait (bounded) for all C chunks of its (sequence, layer,
- * KV head) item, combine their partials (m, Z, O) into this chunk's slice of
- * the output O and the item's per-head (max, 1/Z), turn the unit's stored
- * scores into token masses sum_h exp2(s_hi - max_h) / Z_h (Sec. III-C), then
- * count the chunk as finished.  Run by NT threads, tid < NT: the finisher
- * warp, or all consumer warps for a CTA's last unit.  Returns false, the same
- * for every thread, on abort or timeout.  Loads are issued in batches before
- * the dependent stores, so a pass costs a few L2 round trips. */
-template <int PS, bool ALIGNED, int NT, int OBUF_FLOATS>
-__device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv, int slot, int tid,
-                                            const FinSmem &f) {
-  const float NEG_INF = -INFINITY;
-  const int G = p.G;
+/* The unit's physical page ids (and, with region-aligned pages, their fills)
+ * into shared memory, loaded in batches. */
+template <bool ALIGNED, int NT>
+__device__ __forceinline__ void load_page_ids(const AttnParams &p, const Unit &pv, int tid,
+                                              const FinSmem &f) {
   const int npg = pv.p1 - pv.p0;
-  const int C = pv.C;
-  /* the unit's page ids (no wait needed) */
   const int32_t *bt = p.block_table + (size_t)pv.b * p.P_max;
   for (int q0 = 0; q0 < npg; q0 += NT * 4) {
     int ph[4], fl[4];
@@ -167,6 +161,70 @@ __device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv,
       }
     }
   }
+}
+
+/* Token masses of a unit from its stored raw scores and the item's per-head
+ * (max, 1/Z) in f.fin: mass_i = sum_h exp2(s_hi - max_h) / Z_h, written to
+ * the (layer, KV head) row at the token's physical slot.  Four tokens per
+ * thread in flight (a batch's loads are issued before any store). */
+template <int PS, bool ALIGNED, int NT>
+__device__ __forceinline__ void mass_pass(const AttnParams &p, const Unit &pv, int slot, int tid,
+                                          const FinSmem &f) {
+  const int G = p.G;
+  const int npg = pv.p1 - pv.p0;
+  const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + slot) * p.scratch_tokens * GP;
+  const int ntok = npg * PS;
+  float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
+  float fm[GP], fz[GP];
+#pragma unroll
+  for (int h = 0; h < GP; ++h) {
+    fm[h] = f.fin[h];
+    fz[h] = (h < G) ? f.fin[8 + h] : 0.f;
+  }
+  /* contiguous pages: the valid tokens are a prefix of the unit; with
+   * region-aligned pages every page has its own fill */
+  const int nvalid = ALIGNED ? ntok : min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
+  constexpr int NB = 4;
+  for (int tk0 = 0; tk0 < nvalid; tk0 += NT * NB) {
+    float4 s0[NB], s1[NB];
+#pragma unroll
+    for (int r = 0; r < NB; ++r) {
+      const int tk = tk0 + r * NT + tid;
+      if (tk < nvalid) {
+        s0[r] = __ldcg((const float4 *)(scr + (size_t)tk * GP));
+        s1[r] = __ldcg((const float4 *)(scr + (size_t)tk * GP + 4));
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < NB; ++r) {
+      const int tk = tk0 + r * NT + tid;
+      if (tk >= nvalid) continue;
+      if (ALIGNED && (tk % PS) >= f.sfill[tk / PS]) continue;
+      float m = exp2f(s0[r].x - fm[0]) * fz[0] + exp2f(s0[r].y - fm[1]) * fz[1] +
+                exp2f(s0[r].z - fm[2]) * fz[2] + exp2f(s0[r].w - fm[3]) * fz[3];
+      m += exp2f(s1[r].x - fm[4]) * fz[4] + exp2f(s1[r].y - fm[5]) * fz[5] +
+           exp2f(s1[r].z - fm[6]) * fz[6] + exp2f(s1[r].w - fm[7]) * fz[7];
+      mrow[(size_t)f.sphys[tk / PS] * PS + (tk % PS)] = m;
+    }
+  }
+}
+
+/* The end of a unit: wait (bounded) for all C chunks of its (sequence, layer,
+ * KV head) item, combine their partials (m, Z, O) into this chunk's slice of
+ * the output O and the item's per-head (max, 1/Z), turn the unit's stored
+ * scores into token masses sum_h exp2(s_hi - max_h) / Z_h (Sec. III-C), then
+ * count the chunk as finished.  Run by NT threads, tid < NT: the finisher
+ * warp, or all consumer warps for a CTA's last unit.  Returns false, the same
+ * for every thread, on abort or timeout.  Loads are issued in batches before
+ * the dependent stores, so a pass costs a few L2 round trips. */
+template <int PS, bool ALIGNED, int NT, int OBUF_FLOATS>
+__device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv, int slot, int tid,
+                                            const FinSmem &f) {
+  const float NEG_INF = -INFINITY;
+  const int G = p.G;
+  const int C = pv.C;
+  /* the unit's page ids (no wait needed) */
+  load_page_ids<ALIGNED, NT>(p, pv, tid, f);
   /* all chunks of the item published */
   if (tid == 0) {
     int okw = 1;
@@ -268,51 +326,105 @@ __device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv,
       orow[e] = *(uint16_t *)&bv;
     }
   }
-  /* token masses of this chunk from its stored scores, eight tokens per
-   * thread in flight (a batch's loads are issued before any store) */
-  {
-    const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + slot) * p.scratch_tokens * GP;
-    const int ntok = npg * PS;
-    float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
-    float fm[GP], fz[GP];
-#pragma unroll
-    for (int h = 0; h < GP; ++h) {
-      fm[h] = f.fin[h];
-      fz[h] = (h < G) ? f.fin[8 + h] : 0.f;
-    }
-    /* contiguous pages: the valid tokens are a prefix of the unit; with
-     * region-aligned pages every page has its own fill */
-    const int nvalid = ALIGNED ? ntok : min(ntok, p.n_tokens[pv.b] - pv.p0 * PS);
-    constexpr int NB = 8;
-    for (int tk0 = 0; tk0 < nvalid; tk0 += NT * NB) {
-      float4 s0[NB], s1[NB];
-#pragma unroll
-      for (int r = 0; r < NB; ++r) {
-        const int tk = tk0 + r * NT + tid;
-        if (tk < nvalid) {
-          s0[r] = __ldcg((const float4 *)(scr + (size_t)tk * GP));
-          s1[r] = __ldcg((const float4 *)(scr + (size_t)tk * GP + 4));
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < NB; ++r) {
-        const int tk = tk0 + r * NT + tid;
-        if (tk >= nvalid) continue;
-        if (ALIGNED && (tk % PS) >= f.sfill[tk / PS]) continue;
-        float m = exp2f(s0[r].x - fm[0]) * fz[0] + exp2f(s0[r].y - fm[1]) * fz[1] +
-                  exp2f(s0[r].z - fm[2]) * fz[2] + exp2f(s0[r].w - fm[3]) * fz[3];
-        m += exp2f(s1[r].x - fm[4]) * fz[4] + exp2f(s1[r].y - fm[5]) * fz[5] +
-             exp2f(s1[r].z - fm[6]) * fz[6] + exp2f(s1[r].w - fm[7]) * fz[7];
-        mrow[(size_t)f.sphys[tk / PS] * PS + (tk % PS)] = m;
-      }
-    }
-  }
+  mass_pass<PS, ALIGNED, NT>(p, pv, slot, tid, f);
   fin_sync<NT>();
   if (tid == 0) {
     const int old = atomicAdd(&p.counters[pv.X], 1);
     if (old == 2 * C - 1) atomicExch(&p.counters[pv.X], 0);
   }
   return true;
+}
+
+/* Merge the NCW consumer warps' running softmax states of a unit (per head:
+ * max, sum, O^T) into the chunk's partial (m, Z, O) and publish it: write the
+ * partial, then one gpu-scope fence (cumulative over the threads' writes,
+ * which the sync orders before thread 0) and the item's arrival count.  Run
+ * by NT threads, tid < NT. */
+template <int NCW, int NT>
+__device__ __forceinline__ void merge_publish(const AttnParams &p, const Unit &un, int tid,
+                                              const float *wm, const float *wl, float *wf,
+                                              const float *wO) {
+  const float NEG_INF = -INFINITY;
+  float *part = p.partials + ((size_t)un.X * p.chunk_stride + un.j) * PARTIAL_FLOATS;
+  if (tid < GP) {
+    float M = NEG_INF;
+    for (int w = 0; w < NCW; ++w) M = fmaxf(M, wm[w * 8 + tid]);
+    const float Mr = (M == NEG_INF) ? 0.f : M;
+    float Lsum = 0.f;
+    for (int w = 0; w < NCW; ++w) {
+      const float f = exp2f(wm[w * 8 + tid] - Mr);
+      wf[w * 8 + tid] = f;
+      Lsum += f * wl[w * 8 + tid];
+    }
+    part[tid] = M;
+    part[8 + tid] = Lsum;
+  }
+  fin_sync<NT>();
+  for (int e = tid; e < GP * D; e += NT) {
+    const int h = e >> 7;
+    float acc = 0.f;
+#pragma unroll
+    for (int w = 0; w < NCW; ++w) acc += wf[w * 8 + h] * wO[(size_t)w * GP * D + e];
+    part[16 + e] = acc;
+  }
+  fin_sync<NT>();
+  if (tid == 0) {
+    __threadfence();
+    atomicAdd(&p.counters[un.X], 1);
+  }
+}
+
+/* The end of a unit that is its item's only chunk (C == 1): the merge of
+ * the warps' states is already the item's softmax, so there is no partial,
+ * no counter and no combine.  Writes the per-head (max, 1/Z) to f.fin and
+ * the item's output O, with the same arithmetic (and so the same bits) as
+ * merge_publish followed by finish_unit's combine.  Ends with a sync, after
+ * which the merge buffers are free. */
+template <int NCW, int NT>
+__device__ __forceinline__ void merge_single(const AttnParams &p, const Unit &un, int tid,
+                                             const float *wm, const float *wl, float *wf,
+                                             const float *wO, const FinSmem &f) {
+  const float NEG_INF = -INFINITY;
+  if (tid < GP) {
+    float M = NEG_INF;
+    for (int w = 0; w < NCW; ++w) M = fmaxf(M, wm[w * 8 + tid]);
+    const float Mr = (M == NEG_INF) ? 0.f : M;
+    float Lsum = 0.f;
+    for (int w = 0; w < NCW; ++w) {
+      const float fw = exp2f(wm[w * 8 + tid] - Mr);
+      wf[w * 8 + tid] = fw;
+      Lsum += fw * wl[w * 8 + tid];
+    }
+    f.fin[tid] = Mr;
+    f.fin[8 + tid] = Lsum > 0.f ? 1.f / Lsum : 0.f;
+  }
+  fin_sync<NT>();
+  const int E = p.G * D;
+  uint16_t *orow = p.out + (((size_t)un.b * p.q_layers + (un.l - p.l0)) * p.Hq + (size_t)un.kvh * p.G) * D;
+  for (int e = tid; e < E; e += NT) {
+    const int h = e >> 7;
+    float acc = 0.f;
+#pragma unroll
+    for (int w = 0; w < NCW; ++w) acc += wf[w * 8 + h] * wO[(size_t)w * GP * D + e];
+    acc = f.fin[8 + h] * acc;
+    __nv_bfloat16 bv = __float2bfloat16_rn(acc);
+    orow[e] = *(uint16_t *)&bv;
+  }
+  fin_sync<NT>();
+}
+
+/* The whole end of a single-chunk unit: the page ids, the merge straight
+ * into (max, 1/Z) and the output, the release of the merge buffers (mdone,
+ * when given: the finisher's hand-off), the token masses. */
+template <int PS, bool ALIGNED, int NCW, int NT>
+__device__ __forceinline__ void single_end(const AttnParams &p, const Unit &un, int slot, int tid,
+                                        const float *wm, const float *wl, float *wf,
+                                        const float *wO, const FinSmem &f, uint32_t mdone) {
+  load_page_ids<ALIGNED, NT>(p, un, tid, f);
+  merge_single<NCW, NT>(p, un, tid, wm, wl, wf, wO, f);
+  if (mdone != 0 && tid == 0) mbar_arrive(mdone);   // merge buffers free again
+  mass_pass<PS, ALIGNED, NT>(p, un, slot, tid, f);
+  fin_sync<NT>();
 }
 
 /* ALIGNED: pages carry their own fill (region-aligned allocation); otherwise
@@ -332,7 +444,8 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   uint64_t *qempty = qfull + 2;                         // [2]
   uint64_t *cdone = qempty + 2;    // [2] score slot written, unit published
   uint64_t *fdone = cdone + 2;     // [2] score slot read by the finisher
-  float *wm = (float *)(fdone + 2);           // [NCW][8] per-warp running max
+  uint64_t *mdone = fdone + 2;     // [1] merge buffers read by the finisher
+  float *wm = (float *)(mdone + 2);           // [NCW][8] per-warp running max
   float *wl = wm + NCW * 8;                   // [NCW][8] per-warp running sum
   float *wf = wl + NCW * 8;                   // [NCW][8] per-warp merge factor
   float *wO = wf + NCW * 8;                   // [NCW][8][128] per-warp O^T
@@ -360,9 +473,10 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     for (int s = 0; s < 2; ++s) {
       mbar_init(smem_u32(&qfull[s]), 1);
       mbar_init(smem_u32(&qempty[s]), NCW);
-      mbar_init(smem_u32(&cdone[s]), 1);
+      mbar_init(smem_u32(&cdone[s]), NCW);   // every consumer warp, once per unit
       mbar_init(smem_u32(&fdone[s]), 1);
     }
+    mbar_init(smem_u32(&mdone[0]), 1);
     flag[0] = flag[1] = flag[2] = flag[3] = 0;
     fence_barrier_init();
   }
@@ -376,15 +490,22 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       tma_prefetch_desc(&tmap);
+      /* the i-th page this CTA streams goes to stage i % R, consumed by warp
+       * i % NCW: R is a multiple of NCW, so every stage belongs to one warp */
       int i = 0, nu = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
         const Unit un = decode_unit(p, u);
         /* the unit's G query rows: one bulk copy into a double-buffered slot */
         const int qs = nu & 1;
-        if (nu >= 2 && !wait_phase(smem_u32(&qempty[qs]), ((nu >> 1) - 1) & 1, p, 5, true)) {
-          ok = false;
-          break;
+        if (nu >= 2) {
+          if (!wait_phase(smem_u32(&qempty[qs]), ((nu >> 1) - 1) & 1, p, 5, true)) {
+            ok = false;
+            break;
+          }
+          /* the consumers read the slot through the generic proxy; the bulk
+           * copy writes it through the async proxy */
+          fence_proxy_async_smem();
         }
         mbar_arrive_expect_tx(smem_u32(&qfull[qs]), G * D * 2);
         bulk_load(sQ_u32 + qs * S::Q_BYTES,
@@ -406,10 +527,15 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
           for (int k = 0; k < 8; ++k) {
             if (k >= cnt) break;
             const int s = i % S::R;
-            if (i >= S::R &&
-                !wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
-              ok = false;
-              break;
+            if (i >= S::R) {
+              if (!wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
+                ok = false;
+                break;
+              }
+              /* the stage's last reads (ldmatrix, generic proxy) must be
+               * ordered before the TMA refill (async proxy): without this
+               * fence a refill can overwrite V rows still being read */
+              fence_proxy_async_smem();
             }
             const int row = (((un.l * p.P_phys + ph[k]) * p.Hkv + un.kvh) * 2) * PS;
             const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
@@ -421,7 +547,8 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
           }
         }
       }
-      /* No copy may still be writing this CTA's shared memory when it exits. */
+      /* No copy may still be writing this CTA's shared memory when it exits:
+       * wait for the last copy issued into every stage. */
       for (int k = (i > S::R ? i - S::R : 0); k < i; ++k)
         wait_phase(smem_u32(&full[k % S::R]), (k / S::R) & 1, p, 2, false);
       for (int k = (nu > 2 ? nu - 2 : 0); k < nu; ++k)
@@ -435,14 +562,22 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   if (warp == NCW + 1) {
     /* ------------------------------------------------------- finisher ---- */
     /* The end of every unit but the CTA's last, one warp, while the
-     * consumers stream the next unit; then the score slot is released. */
+     * consumers stream the next unit: merge the warps' states and publish
+     * the chunk's partial, release the merge buffers, finish the unit, then
+     * release its score slot. */
     int k = 0;
     for (int u = blockIdx.x; u < p.total_units; u += gridDim.x, ++k) {
       if (u + (int)gridDim.x >= p.total_units) break;   // the consumers finish the last unit
       const Unit pv = decode_unit(p, u);
       const bool ok = wait_phase(smem_u32(&cdone[k & 1]), (k >> 1) & 1, p, 8, true);
       if (!__all_sync(0xffffffffu, ok)) break;
-      if (!finish_unit<PS, ALIGNED, 32, S::OBUF_FLOATS>(p, pv, k & 1, lane, fs)) break;
+      if (pv.C == 1) {
+        single_end<PS, ALIGNED, NCW, 32>(p, pv, k & 1, lane, wm, wl, wf, wO, fs, smem_u32(&mdone[0]));
+      } else {
+        merge_publish<NCW, 32>(p, pv, lane, wm, wl, wf, wO);
+        if (lane == 0) mbar_arrive(smem_u32(&mdone[0]));   // merge buffers free again
+        if (!finish_unit<PS, ALIGNED, 32, S::OBUF_FLOATS>(p, pv, k & 1, lane, fs)) break;
+      }
       if (lane == 0) mbar_arrive(smem_u32(&fdone[k & 1]));   // slot and finish area free
     }
     return;
@@ -457,8 +592,8 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
   const uint64_t pol_keep = policy_evict_last();
   const float NEG_INF = -INFINITY;
 
-  int i_base = 0, nunit = 0;
-  bool aborted = false;   // this warp gave up a wait
+  int i_base = 0, nunit = 0;   // pages streamed before this unit; units done
+  bool aborted = false;        // this warp gave up a wait
   for (int u = blockIdx.x; u < p.total_units; u += gridDim.x) {
     const Unit un = decode_unit(p, u);
     const int npg = un.p1 - un.p0;
@@ -491,6 +626,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     if (nunit >= 2 && !aborted &&
         !wait_phase(smem_u32(&fdone[slot]), ((nunit >> 1) - 1) & 1, p, 9, true))
       aborted = true;
+    aborted = __any_sync(0xffffffffu, aborted);   // one decision per warp
     float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
     float o[8][4];
 #pragma unroll
@@ -498,7 +634,12 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     const int ntok_seq = p.n_tokens[un.b];
     const int mi = lane >> 3, rr = lane & 7;
 
-    for (int jp = cw; jp < npg && !aborted; jp += NCW) {
+    /* this warp's pages are those whose CTA-wide index gi = i_base + jp is
+     * cw modulo NCW: they land only in this warp's own stages (gi % R), so a
+     * wait is never more than one phase ahead of the copies however far the
+     * warps drift apart, and a unit's extra pages rotate over the warps */
+    const int j0 = ((cw - i_base) % NCW + NCW) % NCW;
+    for (int jp = j0; jp < npg && !aborted; jp += NCW) {
       const int gi = i_base + jp;
       const int s = gi % S::R;
       if (!wait_phase(smem_u32(&full[s]), (gi / S::R) & 1, p, 4, true)) {
@@ -576,19 +717,30 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
     }
 
-    /* ---- merge the warps' partial softmax states, publish the unit's ---- */
+    /* ---- the unit's end: this warp's softmax state goes to the merge ---- */
 #pragma unroll
     for (int off = 4; off < 32; off <<= 1) {
       l0 += __shfl_xor_sync(0xffffffffu, l0, off);
       l1 += __shfl_xor_sync(0xffffffffu, l1, off);
     }
-    if (g == 0) {
-      wm[cw * 8 + 2 * t] = m0;
-      wm[cw * 8 + 2 * t + 1] = m1;
-      wl[cw * 8 + 2 * t] = l0;
-      wl[cw * 8 + 2 * t + 1] = l1;
+    aborted = __any_sync(0xffffffffu, aborted);
+    const bool last = u + (int)gridDim.x >= p.total_units;
+    /* the merge buffers hold the previous unit's states until the finisher
+     * has read them; on the CTA's last unit the finisher must be done with
+     * everything (its finish area is used below) */
+    if (!aborted && nunit >= 1) {
+      const bool okw = last ? wait_phase(smem_u32(&fdone[(nunit - 1) & 1]), ((nunit - 1) >> 1) & 1, p, 9, true)
+                            : wait_phase(smem_u32(&mdone[0]), (nunit - 1) & 1, p, 10, true);
+      if (!okw) aborted = true;
+      aborted = __any_sync(0xffffffffu, aborted);
     }
-    {
+    if (!aborted) {
+      if (g == 0) {
+        wm[cw * 8 + 2 * t] = m0;
+        wm[cw * 8 + 2 * t + 1] = m1;
+        wl[cw * 8 + 2 * t] = l0;
+        wl[cw * 8 + 2 * t + 1] = l1;
+      }
       float *wo = wO + (size_t)cw * GP * D;
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt) {
@@ -598,55 +750,30 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
         wo[(2 * t + 1) * D + 16 * mt + g + 8] = o[mt][3];
       }
     }
+    if (!last) {
+      /* hand the unit to the finisher and go on at once; a warp that gave
+       * up a wait runs on without waiting to the last unit's barrier */
+      __syncwarp();
+      if (!aborted && lane == 0) mbar_arrive(smem_u32(&cdone[slot]));
+      i_base += npg;
+      ++nunit;
+      continue;
+    }
+    /* the CTA's last unit: nothing is left to overlap with, so all consumer
+     * warps merge, publish and finish it */
     if (aborted) flag[0] = 1;
     named_barrier(1, NC);
     if (flag[0]) break;
-    float *part = p.partials + ((size_t)un.X * p.chunk_stride + un.j) * PARTIAL_FLOATS;
-    if (ct < GP) {
-      float M = NEG_INF;
-      for (int w = 0; w < NCW; ++w) M = fmaxf(M, wm[w * 8 + ct]);
-      const float Mr = (M == NEG_INF) ? 0.f : M;
-      float Lsum = 0.f;
-      for (int w = 0; w < NCW; ++w) {
-        const float f = exp2f(wm[w * 8 + ct] - Mr);
-        wf[w * 8 + ct] = f;
-        Lsum += f * wl[w * 8 + ct];
-      }
-      part[ct] = M;
-      part[8 + ct] = Lsum;
-    }
-    named_barrier(1, NC);
-    for (int e = ct; e < GP * D; e += NC) {
-      const int h = e >> 7;
-      float acc = 0.f;
-#pragma unroll
-      for (int w = 0; w < NCW; ++w) acc += wf[w * 8 + h] * wO[(size_t)w * GP * D + e];
-      part[16 + e] = acc;
-    }
-    /* release: the barrier orders every thread's partial (and score) writes
-     * before thread 0, whose gpu-scope fence is cumulative over them */
-    named_barrier(1, NC);
-    if (ct == 0) {
-      __threadfence();
-      atomicAdd(&p.counters[un.X], 1);
-      flag[1] = ld_volatile(&p.status[ST_ABORT]);
-    }
-    named_barrier(1, NC);
-    if (flag[1]) break;
-    if (u + (int)gridDim.x >= p.total_units) {
-      /* the CTA's last unit: nothing is left to overlap with, so all consumer
-       * warps finish it, once the finisher has released the finish area */
-      if (ct == 0)
-        flag[3] = (nunit >= 1 && !wait_phase(smem_u32(&fdone[(nunit - 1) & 1]),
-                                              ((nunit - 1) >> 1) & 1, p, 9, true)) ? 1 : 0;
-      named_barrier(1, NC);
-      if (flag[3]) break;
-      finish_unit<PS, ALIGNED, NCW * 32, S::OBUF_FLOATS>(p, un, slot, ct, fs);
+    if (un.C == 1) {
+      single_end<PS, ALIGNED, NCW, NCW * 32>(p, un, slot, ct, wm, wl, wf, wO, fs, 0u);
       break;
     }
-    if (ct == 0) mbar_arrive(smem_u32(&cdone[slot]));   // hand the unit to the finisher
-    i_base += npg;
-    ++nunit;
+    merge_publish<NCW, NCW * 32>(p, un, ct, wm, wl, wf, wO);
+    if (ct == 0) flag[1] = ld_volatile(&p.status[ST_ABORT]);
+    named_barrier(1, NC);
+    if (flag[1]) break;
+    finish_unit<PS, ALIGNED, NCW * 32, S::OBUF_FLOATS>(p, un, slot, ct, fs);
+    break;
   }
 }
 

@@ -30,6 +30,13 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
+/* Orders this CTA's earlier generic-proxy shared-memory accesses (the ones
+ * made visible to this thread by an mbarrier acquire included) before later
+ * async-proxy accesses: a stage or slot that consumers read with ldmatrix must
+ * not be refilled by a TMA / bulk copy until this fence has been issued. */
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }

@@ -231,6 +231,54 @@ def test_bit_identical_reruns():
         assert torch.equal(x, y)
 
 
+def test_config2_full_trace_step_is_bit_identical_over_reruns():
+    """The full-trace step of the 3B geometry (32 x 1,700 tokens, one split per
+    (sequence, layer, KV head), several units per CTA) repeated from one saved
+    state gives bit-identical outputs and mass rows.  A ring stage refilled by
+    TMA (async proxy) before the consumers' ldmatrix reads of it (generic
+    proxy) were fenced showed up here as rare, small differences in one
+    item's output (its V rows read after the refill had begun)."""
+    w = synth.make_workload(2)
+    dev = torch.device("cuda")
+    B, L, Hq, Hkv, D = w.B, w.L, w.Hq, w.Hkv, w.D
+    c = md.Cache(L, Hq, Hkv, w.page_size, B, w.max_pages_per_seq(), w.num_phys_pages())
+    for r in range(7):
+        c.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    lib = synth.lib()
+    nmax = max(w.n0(b) for b in range(B))
+    kb = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
+    vb = torch.empty_like(kb)
+    for b in range(B):
+        rd = torch.from_numpy(w.regions[b]).to(dev)
+        assert lib.synth_fill_kv_dev(w.seed, 0, None, b, L, Hkv, D, 0, w.n0(b), rd.data_ptr(),
+                                     kb.data_ptr(), vb.data_ptr(), None) == 0
+        c.append_tokens(b, w.regions[b], kb.data_ptr(), vb.data_ptr(), w.insert_steps[b])
+    q = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+    kn = torch.empty((B, L, Hkv, D), dtype=torch.int16, device=dev)
+    vn = torch.empty_like(kn)
+    pos = torch.tensor([w.n0(b) for b in range(B)], dtype=torch.int32, device=dev)
+    rg = torch.tensor([w.decode_region] * B, dtype=torch.uint8, device=dev)
+    assert lib.synth_fill_q_dev(w.seed, 0, None, B, L, Hq, Hq // Hkv, D, 1, q.data_ptr(), None) == 0
+    assert lib.synth_fill_step_kv_dev(w.seed, 0, None, B, L, Hkv, D, pos.data_ptr(), rg.data_ptr(),
+                                      kn.data_ptr(), vn.data_ptr(), None) == 0
+    torch.cuda.synchronize()
+    saved = c.save_state()
+    ref = None
+    for rep in range(16):
+        c.load_state(saved)
+        out = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+        c.decode_step(B, q, kn, vn, [w.decode_region] * B, out)
+        got = (out.clone(), c.get_state(md.MD_STATE_MASS).clone())
+        torch.cuda.synchronize()
+        if ref is None:
+            ref = got
+            continue
+        assert torch.equal(got[0], ref[0]), f"attention output differs on rerun {rep}"
+        assert torch.equal(got[1], ref[1]), f"mass rows differ on rerun {rep}"
+    assert c.sync() == md.MD_OK
+    c.close()
+
+
 def test_checkpoint_restore_replays_step():
     w = synth.custom_workload("ckpt", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900],
                               budget_frac=0.3, steps=2, seed=9)

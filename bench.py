@@ -364,7 +364,10 @@ def _oracle_worker(task):
     return out
 
 
-def parallel_oracle(args, reps: int, layers: int = 1):
+ORACLE_SAMPLE_LAYERS = 8   # layers of the oracle's bounded sample (a few seconds per process)
+
+
+def parallel_oracle(args, reps: int, layers: int = ORACLE_SAMPLE_LAYERS):
     """Time the fp64 oracle on the host cores: one process per core (numpy
     single-threaded in each), each on its own sequence of the workload.  The
     whole workload's step time is ceil(B / P) times the slowest process's
@@ -373,6 +376,7 @@ def parallel_oracle(args, reps: int, layers: int = 1):
     processes, sample text)."""
     import multiprocessing as mp
     w = make_workload(args, args.seed)
+    layers = max(1, min(layers, w.L))
     try:
         ncpu = len(os.sched_getaffinity(0))
     except AttributeError:
@@ -392,7 +396,7 @@ def parallel_oracle(args, reps: int, layers: int = 1):
         per_rep.append(rounds * slowest)
     sample = (f"sequences 0..{P - 1} of {w.B}, one per process on {P} host cores (single-threaded "
               f"numpy), {layers} of {w.L} layers of the full trace ({w.n0(0)} tokens each): decode time "
-              f"x{w.L // layers} layers + observation/eviction, x{rounds} rounds")
+              f"x{w.L / layers:g} + observation/eviction, x{rounds} rounds")
     return per_rep, P, sample
 
 
@@ -499,7 +503,7 @@ def main():
                        "ms_per_step": e["ms_per_step"], "h2d_bytes_per_step": e["h2d_bytes_per_step"],
                        "d2h_bytes_per_step": e["d2h_bytes_per_step"]}
     if not args.no_cpu_baseline and world == 1:
-        per_rep, cores, sample = parallel_oracle(args, 2)
+        per_rep, cores, sample = parallel_oracle(args, 3)
         line["cpu_baseline"] = {"value": sum(w.n0(b) + 1 for b in range(w.B)) / min(per_rep), "unit": UNIT,
                                 "cores": cores, "kind": "oracle", "sample": sample}
     print(json.dumps(line), flush=True)

@@ -255,11 +255,31 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
   }
 }
 
+/* Blocks of the score kernel that are resident at once on the current device
+ * (SMs x blocks per SM from the occupancy of the instance).  The kernel gives
+ * every block an equal share of the pages, so a grid larger than one wave
+ * would leave the second wave's blocks as a tail. */
+template <int PS>
+static int score_grid_cap() {
+  static int cached[64];   // per device ordinal; a racy first fill writes the same value
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152 * 4;
+  if (cached[dev] > 0) return cached[dev];
+  int sms = 0, per_sm = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_kernel<PS>, 256, 0) != cudaSuccess ||
+      sms <= 0 || per_sm <= 0)
+    return 152 * 4;
+  cached[dev] = sms * per_sm;
+  return cached[dev];
+}
+
 cudaError_t launch_score(const ScoreParams &p, cudaStream_t s) {
   if (p.total_pages == 0) return cudaSuccess;
   const int ppb = 256 / p.ps;
   long long blocks = (p.total_pages + ppb - 1) / ppb;
-  if (blocks > 152 * 8) blocks = 152 * 8;
+  const int cap = p.ps == 16 ? score_grid_cap<16>() : score_grid_cap<32>();
+  if (blocks > cap) blocks = cap;
   if (p.ps == 16) score_kernel<16><<<(int)blocks, 256, 0, s>>>(p);
   else score_kernel<32><<<(int)blocks, 256, 0, s>>>(p);
   return cudaGetLastError();

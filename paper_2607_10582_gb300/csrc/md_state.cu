@@ -367,14 +367,38 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
       if (k != KEY_PINNED && (k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int k = s_k, cum = 0, digit = -1;
-      for (int dgt = 0; dgt < 256; ++dgt) {
-        if (cum + hist[dgt] >= k) { digit = dgt; break; }
-        cum += hist[dgt];
+    if (threadIdx.x < 32) {
+      /* the digit holding the k-th smallest remaining key: one warp, eight
+       * bins per lane; the lane whose cumulative range (excl, incl] holds k
+       * walks its bins (the same digit and residual a serial scan finds) */
+      const int lane = threadIdx.x;
+      const int k = s_k;
+      int c[8], sum = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c[j] = hist[lane * 8 + j];
+        sum += c[j];
       }
-      if (digit < 0) s_bad = 1;           // fewer evictable pages than e
-      else { s_prefix = prefix | ((uint32_t)digit << shift); s_k = k - cum; }
+      int incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const int excl = incl - sum;
+      const bool mine = excl < k && k <= incl;
+      if (__ballot_sync(0xffffffffu, mine) == 0u) {
+        if (lane == 0) s_bad = 1;         // fewer evictable pages than e
+      } else if (mine) {
+        int cum = excl, digit = lane * 8;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (cum + c[j] >= k) { digit = lane * 8 + j; break; }
+          cum += c[j];
+        }
+        s_prefix = prefix | ((uint32_t)digit << shift);
+        s_k = k - cum;
+      }
     }
     __syncthreads();
     if (s_bad) {
@@ -429,9 +453,18 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
 cudaError_t launch_select(const SelectParams &p, cudaStream_t s) {
   if (p.n_seqs == 0) return cudaSuccess;
   const size_t smem = (size_t)p.P_max * 9;
-  cudaError_t err = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+  /* raise the kernel's dynamic shared-memory limit only when a larger table
+   * needs it (a host call per launch costs more than the kernel at small
+   * sizes); per device ordinal, a racy first fill sets the same value */
+  static int granted[64];
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
+  if (dev < 0 || dev >= 64 || granted[dev] < (int)smem) {
+    err = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (err != cudaSuccess) return err;
+    if (dev >= 0 && dev < 64) granted[dev] = (int)smem;
+  }
   select_kernel<<<p.n_seqs, SEL_THREADS, smem, s>>>(p);
   return cudaGetLastError();
 }

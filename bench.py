@@ -294,10 +294,17 @@ def run_native(args, rank, world, local_rank):
                 cache.load_state(saved)
             torch.cuda.synchronize()
             t0 = time.perf_counter()
-            for d_t, h_t in zip(step_inputs, hosts):
-                d_t.copy_(h_t, non_blocking=True)
-            one_step()
-            outh.copy_(step_output, non_blocking=True)
+            if args.layerwise:
+                # the per-layer entry takes device tensors: copy in, run, copy out
+                for d_t, h_t in zip(step_inputs, hosts):
+                    d_t.copy_(h_t, non_blocking=True)
+                one_step()
+                outh.copy_(step_output, non_blocking=True)
+            else:
+                # the host-buffer entry point copies inputs and output itself
+                cache.decode_step_host(B, hosts[0], hosts[1], hosts[2], regs, outh)
+                if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
+                    cache.evict(budgets)
             torch.cuda.synchronize()
             if i >= args.warmup:
                 e_ms.append((time.perf_counter() - t0) * 1e3)
@@ -501,7 +508,9 @@ def main():
         e = r["e2e"]
         line["e2e"] = {"value": e["tokens_per_step"] * world / (e["ms_per_step"] / 1e3), "unit": UNIT,
                        "ms_per_step": e["ms_per_step"], "h2d_bytes_per_step": e["h2d_bytes_per_step"],
-                       "d2h_bytes_per_step": e["d2h_bytes_per_step"]}
+                       "d2h_bytes_per_step": e["d2h_bytes_per_step"],
+                       "entry": ("pinned-host copies + md_decode_layer x L + md_evict" if args.layerwise
+                                 else "md_decode_step_host (host buffers, copies in the call) + md_evict")}
     if not args.no_cpu_baseline and world == 1:
         per_rep, cores, sample = parallel_oracle(args, 3)
         line["cpu_baseline"] = {"value": sum(w.n0(b) + 1 for b in range(w.B)) / min(per_rep), "unit": UNIT,

@@ -162,6 +162,23 @@ md_status md_append_tokens(md_ctx *ctx, int seq, int n_tokens, const uint8_t *re
 md_status md_decode_step(md_ctx *ctx, int batch, const void *q_dev, const void *k_new_dev,
                          const void *v_new_dev, const uint8_t *new_region_host, void *out_dev);
 
+/* md_decode_step with the step's tensors in host memory: the query rows and
+ * the new tokens' K/V are copied into the workspace, the step runs, and the
+ * output is copied back, all enqueued on the handle's stream in that order.
+ * Like every call it is asynchronous: out_host holds the output once the
+ * stream has reached the copy (md_sync, or a synchronisation of the
+ * stream), and the input buffers must stay unchanged until then.  Pinned
+ * (page-locked) host memory gives full copy speed; pageable memory works,
+ * with the copies then partly synchronous.  Layouts as md_decode_step:
+ *   q_host                  bf16 [batch][L][Hq][D]   (host)
+ *   k_new_host, v_new_host  bf16 [batch][L][Hkv][D]  (host)
+ *   new_region_host         [batch]                  (host)
+ *   out_host                bf16 [batch][L][Hq][D]   (host, written)
+ * Errors as md_decode_step; every argument check runs before any copy. */
+md_status md_decode_step_host(md_ctx *ctx, int batch, const void *q_host, const void *k_new_host,
+                              const void *v_new_host, const uint8_t *new_region_host,
+                              void *out_host);
+
 /* The same decode step, one layer per call, for a model that runs its other
  * per-layer work (MLP, norms) between the layers' attentions: the production
  * shape of the loop (Fig. 1: the decode engine appends KV and attends layer

@@ -71,6 +71,7 @@ SIGNATURES = {
     "md_set_region_params": (_c.c_int, [_P, _c.c_int, _c.c_float, _c.c_float, _c.c_int]),
     "md_append_tokens": (_c.c_int, [_P, _c.c_int, _c.c_int, _P, _P, _P, _P]),
     "md_decode_step": (_c.c_int, [_P, _c.c_int, _P, _P, _P, _P, _P]),
+    "md_decode_step_host": (_c.c_int, [_P, _c.c_int, _P, _P, _P, _P, _P]),
     "md_decode_layer": (_c.c_int, [_P, _c.c_int, _c.c_int, _P, _P, _P, _P, _P]),
     "md_evict": (_c.c_int, [_P, _c.c_int, _P, _P, _P]),
     "md_sync": (_c.c_int, [_P]),
@@ -124,6 +125,18 @@ def _ptr(x) -> Optional[int]:
         return None
     if isinstance(x, int):
         return x
+    return x.data_ptr()
+
+
+def _hptr(x) -> int:
+    """Address of a contiguous host buffer: a CPU torch tensor (pinned for
+    full copy speed) or a numpy array."""
+    if isinstance(x, np.ndarray):
+        if not x.flags["C_CONTIGUOUS"]:
+            raise ValueError("host buffer must be contiguous")
+        return x.ctypes.data
+    if x.is_cuda or not x.is_contiguous():
+        raise ValueError("host buffer must be a contiguous CPU tensor")
     return x.data_ptr()
 
 
@@ -219,6 +232,14 @@ class Cache:
     def decode_step(self, batch: int, q, k_new, v_new, new_regions, out):
         regs, rp = _host(new_regions, np.uint8)
         return self._check(lib().md_decode_step(self.h, batch, _ptr(q), _ptr(k_new), _ptr(v_new), rp, _ptr(out)))
+
+    def decode_step_host(self, batch: int, q, k_new, v_new, new_regions, out):
+        """md_decode_step_host: q, k_new, v_new and out are host buffers (CPU
+        tensors or numpy arrays, bf16 bits); out is written once the stream
+        gets there (sync() or a stream synchronisation)."""
+        regs, rp = _host(new_regions, np.uint8)
+        return self._check(lib().md_decode_step_host(self.h, batch, _hptr(q), _hptr(k_new), _hptr(v_new), rp,
+                                                     _hptr(out)))
 
     def decode_layer(self, layer: int, batch: int, q, k_new, v_new, new_regions, out):
         regs, rp = _host(new_regions, np.uint8)

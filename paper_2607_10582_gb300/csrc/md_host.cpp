@@ -401,6 +401,13 @@ size_t md::compute_layout(const md_config &c, Layout *lay) {
   L.page_fill = take((size_t)c.max_batch * c.max_pages_per_seq, 256);
   L.seq_tokens = take((size_t)c.max_batch * 4, 256);
   L.calib = take((size_t)8 * CALIB_BUCKETS * (8 + 4), 256);
+  /* device copies of one step's tensors for md_decode_step_host */
+  const size_t q_bytes = (size_t)c.max_batch * c.num_layers * c.num_q_heads * D * 2;
+  const size_t kv_bytes = (size_t)c.max_batch * c.num_layers * c.num_kv_heads * D * 2;
+  L.io_q = take(q_bytes, 256);
+  L.io_k = take(kv_bytes, 256);
+  L.io_v = take(kv_bytes, 256);
+  L.io_out = take(q_bytes, 256);
   L.total = align_up(off, 256);
   if (lay) *lay = L;
   return L.total;
@@ -762,6 +769,34 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   st = run_attention(c, batch, 0, cf.num_layers, cf.num_layers, q_dev, out_dev);
   if (st != MD_OK) return st;
   end_step(c, batch);
+  return MD_OK;
+}
+
+MD_API md_status md_decode_step_host(md_ctx *c, int batch, const void *q_host, const void *k_new_host,
+                                     const void *v_new_host, const uint8_t *new_region_host,
+                                     void *out_host) {
+  if (!c) return MD_ERR_INVALID_ARG;
+  if (c->poisoned) return fail(c, MD_ERR_STATE, "handle unusable after an earlier error");
+  if (c->m.layer_next != 0) return fail(c, MD_ERR_STATE, "a layer-by-layer step is in progress");
+  if (!q_host || !k_new_host || !v_new_host || !out_host)
+    return fail(c, MD_ERR_INVALID_ARG, "null pointer");
+  /* every check of the step before anything is copied: the copies are sized
+   * by batch, which must fit the workspace */
+  md_status st = check_step(c, batch, new_region_host);
+  if (st != MD_OK) return st;
+  const md_config &cf = c->cfg;
+  const size_t q_bytes = (size_t)batch * cf.num_layers * cf.num_q_heads * D * 2;
+  const size_t kv_bytes = (size_t)batch * cf.num_layers * cf.num_kv_heads * D * 2;
+  uint8_t *dq = c->ws + c->lay.io_q, *dk = c->ws + c->lay.io_k, *dv = c->ws + c->lay.io_v,
+          *dout = c->ws + c->lay.io_out;
+  cudaError_t e = cudaMemcpyAsync(dq, q_host, q_bytes, cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(dk, k_new_host, kv_bytes, cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(dv, v_new_host, kv_bytes, cudaMemcpyHostToDevice, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "input copy");
+  st = md_decode_step(c, batch, dq, dk, dv, new_region_host, dout);
+  if (st != MD_OK) return st;
+  e = cudaMemcpyAsync(out_host, dout, q_bytes, cudaMemcpyDeviceToHost, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "output copy");
   return MD_OK;
 }
 

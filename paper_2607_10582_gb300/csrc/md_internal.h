@@ -31,7 +31,7 @@ struct RegionTable {
 struct Layout {
   size_t pool, block_table, page_score, free_stack, region, a, t_ref, t_ins, window, ahat, prio, mass,
       scratch, partials, counters, evict_list, staging_regions, staging_steps, staging_slots, status,
-      calib, page_fill, seq_tokens, total;
+      calib, page_fill, seq_tokens, io_q, io_k, io_v, io_out, total;
   size_t slots, n_items;
   int scratch_tokens, chunk_stride;
 };

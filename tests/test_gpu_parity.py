@@ -279,6 +279,51 @@ def test_config2_full_trace_step_is_bit_identical_over_reruns():
     c.close()
 
 
+def test_decode_step_host_matches_device_path():
+    """md_decode_step_host (host buffers; the copies are enqueued inside the
+    call) gives the same bits as md_decode_step from the same state, with
+    pinned torch tensors and with pageable numpy arrays; an out-of-range batch
+    is rejected before anything is copied."""
+    w = synth.custom_workload("host", L=2, Hq=16, Hkv=2, page_size=16, lengths=[700, 1500],
+                              budget_frac=0.5, steps=4, seed=5, structured=True)
+    B, L, Hq, Hkv = w.B, w.L, w.Hq, w.Hkv
+    c = md.Cache(L, Hq, Hkv, w.page_size, B, w.max_pages_per_seq(), w.num_phys_pages())
+    for r in range(7):
+        c.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+    for b in range(B):
+        k, v = synth.kv_host(w.seed, b, L, Hkv, 0, w.n0(b), w.regions[b], True)
+        c.append_tokens(b, w.regions[b], to_dev(k), to_dev(v))
+    q = np.ascontiguousarray(synth.q_host(w.seed, B, L, Hq, Hkv, 1, True))
+    kn, vn = (np.ascontiguousarray(x) for x in
+              synth.step_kv_host(w.seed, [w.n0(b) for b in range(B)], [6] * B, L, Hkv, True))
+    regs = [6] * B
+    torch.cuda.synchronize()
+    saved = c.save_state()
+    out_dev = torch.empty((B, L, Hq, 128), dtype=torch.int16, device="cuda")
+    c.decode_step(B, to_dev(q), to_dev(kn), to_dev(vn), regs, out_dev)
+    ref_o = out_dev.cpu()
+    ref_m = c.get_state(md.MD_STATE_MASS).cpu()
+
+    c.load_state(saved)
+    qh, kh, vh = (torch.from_numpy(x.view(np.int16)).pin_memory() for x in (q, kn, vn))
+    outh = torch.zeros((B, L, Hq, 128), dtype=torch.int16).pin_memory()
+    c.decode_step_host(B, qh, kh, vh, regs, outh)
+    assert c.sync() == md.MD_OK
+    assert torch.equal(outh, ref_o)
+    assert torch.equal(c.get_state(md.MD_STATE_MASS).cpu(), ref_m)
+
+    c.load_state(saved)
+    outn = np.zeros((B, L, Hq, 128), np.uint16)
+    c.decode_step_host(B, q, kn, vn, regs, outn)
+    assert c.sync() == md.MD_OK
+    assert np.array_equal(outn, ref_o.numpy().view(np.uint16))
+
+    with pytest.raises(md.MemDecayError) as ei:
+        c.decode_step_host(B + 1, q, kn, vn, regs + [6], outn)
+    assert ei.value.status == md.MD_ERR_INVALID_ARG
+    c.close()
+
+
 def test_checkpoint_restore_replays_step():
     w = synth.custom_workload("ckpt", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900],
                               budget_frac=0.3, steps=2, seed=9)

@@ -239,7 +239,10 @@ enum {
   MD_STATE_POOL = 10,       /* bf16  [L][num_phys_pages][Hkv][2][page_size][D] K/V    */
   MD_STATE_T_INS = 11,      /* int32 [slots] insertion step                           */
   MD_STATE_PAGE_FILL = 12,  /* uint8 [max_batch][max_pages_per_seq] tokens per page   */
-  MD_STATE_SEQ_TOKENS = 13  /* int32 [max_batch] tokens per sequence (device count)   */
+  MD_STATE_SEQ_TOKENS = 13, /* int32 [max_batch] tokens per sequence (device count)   */
+  MD_STATE_CALIB = 14       /* bytes: the calibration histogram, u64 [8][MD_CALIB_BUCKETS]
+                               fixed-point mass sums (2^32 = 1.0), then u32 [8][MD_CALIB_BUCKETS]
+                               counts; part of a checkpoint                            */
 };
 
 /* Device-to-device copy of one state array into dst_dev (bytes must equal the

@@ -37,7 +37,7 @@ MD_HEAD_DIM = 128
 
 (MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A, MD_STATE_T_REF,
  MD_STATE_AHAT, MD_STATE_FREE, MD_STATE_REGION, MD_STATE_WINDOW, MD_STATE_MASS, MD_STATE_POOL,
- MD_STATE_T_INS, MD_STATE_PAGE_FILL, MD_STATE_SEQ_TOKENS) = range(14)
+ MD_STATE_T_INS, MD_STATE_PAGE_FILL, MD_STATE_SEQ_TOKENS, MD_STATE_CALIB) = range(15)
 MD_CALIB_BUCKETS = 256
 MD_CALIB_BUCKET_WIDTH = 4
 (MD_QUERY_TOKENS, MD_QUERY_PAGES, MD_QUERY_FREE_TOP, MD_QUERY_STEP, MD_QUERY_WINDOW,
@@ -279,6 +279,7 @@ class Cache:
             MD_STATE_T_INS: ((slots,), t.int32),
             MD_STATE_PAGE_FILL: ((self.max_batch, self.P_max), t.uint8),
             MD_STATE_SEQ_TOKENS: ((self.max_batch,), t.int32),
+            MD_STATE_CALIB: ((8 * MD_CALIB_BUCKETS * 12,), t.uint8),
         }[what]
 
     def get_state(self, what: int):

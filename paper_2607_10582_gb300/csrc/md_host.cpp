@@ -1026,6 +1026,7 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
       *bytes = (size_t)cf.max_batch * cf.max_pages_per_seq;
       return true;
     case MD_STATE_SEQ_TOKENS: *off = L.seq_tokens; *bytes = (size_t)cf.max_batch * 4; return true;
+    case MD_STATE_CALIB: *off = L.calib; *bytes = (size_t)8 * CALIB_BUCKETS * (8 + 4); return true;
     case MD_STATE_POOL:
       *off = L.pool;
       *bytes = (size_t)cf.num_layers * cf.num_phys_pages * cf.num_kv_heads * 2 * cf.page_size * D * 2;
@@ -1035,7 +1036,8 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
 }
 const int SAVED[] = {MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A,
                      MD_STATE_T_REF,       MD_STATE_AHAT,       MD_STATE_FREE,       MD_STATE_REGION,
-                     MD_STATE_WINDOW,      MD_STATE_T_INS,      MD_STATE_PAGE_FILL,  MD_STATE_SEQ_TOKENS};
+                     MD_STATE_WINDOW,      MD_STATE_T_INS,      MD_STATE_PAGE_FILL,  MD_STATE_SEQ_TOKENS,
+                     MD_STATE_CALIB};
 }  // namespace
 
 MD_API md_status md_get_state(md_ctx *c, int what, void *dst, size_t bytes) {
@@ -1089,7 +1091,7 @@ MD_API md_status md_query(const md_ctx *c, int what, int seq, int64_t *out) {
 namespace {
 size_t host_blob_bytes(const md_ctx *c) {
   const size_t B = c->cfg.max_batch;
-  return sizeof(HostMirror) + sizeof(RegionTable) + B * (8 + 4 + 4 + 1 + 4 + 4 + 1);
+  return sizeof(HostMirror) + sizeof(RegionTable) + B * (8 + 4 + 4 + 1 + 4 + 4 + 1) + 1;
 }
 }  // namespace
 
@@ -1136,6 +1138,8 @@ MD_API md_status md_save_state(md_ctx *c, void *dst_dev, void *host_blob) {
   memcpy(h, c->tail_region.data(), B * 4);
   h += B * 4;
   memcpy(h, c->tokens_exact.data(), B);
+  h += B;
+  *h = c->calib_on ? 1 : 0;
   return MD_OK;
 }
 
@@ -1169,6 +1173,8 @@ MD_API md_status md_load_state(md_ctx *c, const void *src_dev, const void *host_
   memcpy(c->tail_region.data(), h, B * 4);
   h += B * 4;
   memcpy(c->tokens_exact.data(), h, B);
+  h += B;
+  c->calib_on = *h != 0;
   return MD_OK;
 }
 

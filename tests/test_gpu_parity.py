@@ -347,6 +347,35 @@ def test_checkpoint_restore_replays_step():
         assert torch.equal(x, y)
 
 
+def test_checkpoint_carries_the_calibration_histogram():
+    """A checkpoint taken with calibration on restores the histogram (and the
+    switch): replaying a step from it gives the same histogram as the first
+    time, whatever was gathered in between."""
+    w = synth.custom_workload("ckcal", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900, 400],
+                              budget_frac=0.4, steps=4, seed=13, structured=True)
+    ls = Lockstep(w)
+    ls.prefill()
+    ls.gpu.calib_enable(True)
+    ls.decode()
+    ls.observe()
+    saved = ls.gpu.save_state()
+    q = synth.q_host(w.seed, w.B, w.L, w.Hq, w.Hkv, 7, True)
+    kn, vn = synth.step_kv_host(w.seed, [5000, 5000], [6, 6], w.L, w.Hkv, True)
+    res = []
+    for _ in range(2):
+        ls.gpu.load_state(saved)
+        out = torch.empty((w.B, w.L, w.Hq, 128), dtype=torch.int16, device="cuda")
+        ls.gpu.decode_step(w.B, to_dev(q), to_dev(kn), to_dev(vn), [6, 6], out)
+        ls.gpu.evict(w.budget_pages)
+        s, n = ls.gpu.calib_read()
+        res.append((np.array(s), np.array(n)))
+        # gather more in between: the restore must undo it
+        ls.gpu.decode_step(w.B, to_dev(q), to_dev(kn), to_dev(vn), [6, 6], out)
+        ls.gpu.evict(w.budget_pages)
+    assert np.array_equal(res[0][0], res[1][0]) and np.array_equal(res[0][1], res[1][1])
+    assert res[0][1].sum() > 0
+
+
 def test_capacity_and_argument_errors_are_synchronous():
     c = md.Cache(1, 8, 2, 16, 2, 4, 6)
     k = torch.zeros((1, 2, 80, 128), dtype=torch.int16, device="cuda")

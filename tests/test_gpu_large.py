@@ -1,7 +1,9 @@
 """Full-size parity at configs 3 and 4, in the benchmark's launch
 configuration (the whole batch, 77 GB of K/V per step, on the GPU), checked
 on sampled sequences {0, B/2, B-1} that the oracle recomputes one by one: at
-the full-trace observation and at the steady observations after it.
+the full-trace observation and at the steady observations after it.  Config 4
+is also run through the layer-by-layer entry point and with region-aligned
+pages (pages then hold different numbers of tokens).
 
 Sequences are independent in every stage except the shared page pool, so the
 oracle runs a sampled sequence alone (its physical page ids differ) and the
@@ -30,15 +32,28 @@ mdbuild.build()
 synth.build()
 
 
-def gpu_run(w, n_obs, samples):
+def sizes(w, aligned):
+    """Block-table width and pool size; region-aligned pages may leave one
+    partly filled page per region span (and one more for the decode tokens)."""
+    P_max, P_phys = w.max_pages_per_seq(), w.num_phys_pages()
+    if aligned:
+        spans = [int(np.count_nonzero(np.diff(w.regions[b].astype(np.int16)))) + 2 for b in range(w.B)]
+        P_max += max(spans)
+        P_phys += sum(spans)
+    return P_max, P_phys
+
+
+def gpu_run(w, n_obs, samples, mode="fused"):
     """Prefill the whole batch with the CUDA generator, then n_obs observation
     windows of window_k decode steps each; keep, for the sampled sequences,
     what each observation needs for the comparison."""
     dev = torch.device("cuda")
     B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
-    cache = md.Cache(L, Hq, Hkv, ps, B, w.max_pages_per_seq(), w.num_phys_pages(),
+    P_max, P_phys = sizes(w, mode == "aligned")
+    cache = md.Cache(L, Hq, Hkv, ps, B, P_max, P_phys,
                      rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
-                     score_mode=w.score_mode, page_reduce=w.page_reduce)
+                     score_mode=w.score_mode, page_reduce=w.page_reduce,
+                     region_aligned_pages=int(mode == "aligned"))
     for r in range(7):
         cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
     lib = synth.lib()
@@ -67,9 +82,19 @@ def gpu_run(w, n_obs, samples):
             assert lib.synth_fill_q_dev(w.seed, 0, None, B, L, Hq, Hq // Hkv, D, t, q.data_ptr(), None) == 0
             assert lib.synth_fill_step_kv_dev(w.seed, 0, None, B, L, Hkv, D, pos.data_ptr(), rdev.data_ptr(),
                                               kn.data_ptr(), vn.data_ptr(), None) == 0
-            cache.decode_step(B, q, kn, vn, regs, out)
+            if mode == "layerwise":
+                # a model hands each layer its own contiguous [B][heads][D] tensors
+                for l in range(L):
+                    ol = torch.empty((B, Hq, D), dtype=torch.int16, device=dev)
+                    cache.decode_layer(l, B, q[:, l].contiguous(), kn[:, l].contiguous(),
+                                       vn[:, l].contiguous(), regs, ol)
+                    out[:, l] = ol
+            else:
+                cache.decode_step(B, q, kn, vn, regs, out)
         o_last = out.cpu().numpy().view(np.uint16)
         pre_bt = cache.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
+        pre_fill = cache.get_state(md.MD_STATE_PAGE_FILL).cpu().numpy()
+        pre_pages = [cache.query(md.MD_QUERY_PAGES, b) for b in range(B)]
         pre_tokens = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
         st, n_ev = cache.evict(w.budget_pages)
         torch.cuda.synchronize()
@@ -81,8 +106,10 @@ def gpu_run(w, n_obs, samples):
         rec = {}
         for b in samples:
             n_pre = pre_tokens[b]
-            gsl = np.array([pre_bt[b, i // ps] * ps + i % ps for i in range(n_pre)])
-            P = -(-n_pre // ps)
+            P = pre_pages[b]
+            fills = [int(pre_fill[b, j]) if mode == "aligned" else min(ps, n_pre - j * ps) for j in range(P)]
+            gsl = np.array([pre_bt[b, j] * ps + o for j in range(P) for o in range(fills[j])])
+            assert len(gsl) == n_pre
             rec[b] = dict(n_ev=int(n_ev[b]), n_pre=n_pre, out=o_last[b].copy(), pre_bt=pre_bt[b, :P].copy(),
                           ahat=st_arr["ahat"][gsl], a=st_arr["a"][gsl], t_ref=st_arr["t_ref"][gsl],
                           prio=st_arr["prio"][gsl], page=st_arr["page"][b, :P].copy(),
@@ -96,14 +123,16 @@ def gpu_run(w, n_obs, samples):
     return obs
 
 
-def oracle_run(w, b, n_obs):
+def oracle_run(w, b, n_obs, aligned=False):
     """The oracle for sequence b alone, same inputs, same schedule; yields one
     record per observation."""
     n = w.n0(b)
-    cfg = om.OracleConfig(w.L, w.Hq, w.Hkv, w.D, w.page_size, 1, w.max_pages_per_seq(),
-                          w.pages0(b) + n_obs * w.window_k // w.page_size + 2, rho=w.rho, gamma=w.gamma,
+    P_max, _ = sizes(w, aligned)
+    spans = int(np.count_nonzero(np.diff(w.regions[b].astype(np.int16)))) + 2 if aligned else 0
+    cfg = om.OracleConfig(w.L, w.Hq, w.Hkv, w.D, w.page_size, 1, P_max,
+                          w.pages0(b) + n_obs * w.window_k // w.page_size + 2 + spans, rho=w.rho, gamma=w.gamma,
                           tau_scale=w.tau_scale, attn_weight=w.attn_weight, score_mode=w.score_mode,
-                          page_reduce=w.page_reduce)
+                          page_reduce=w.page_reduce, region_aligned=aligned)
     o = om.Oracle(cfg)
     for r in range(7):
         o.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
@@ -119,11 +148,12 @@ def oracle_run(w, b, n_obs):
             O = o.decode_step(1, q, kn[:, :, 0, :][None], vn[:, :, 0, :][None], [w.decode_region])
         pre_block = list(o.block[0])
         pre_slots = o.slots(0)
+        pre_pot = o.page_of_token(0)
         st, n_ev, ids, logical = o.evict(1, [w.budget_pages[b]])
-        yield o, O[0], pre_block, pre_slots, n_ev[0], logical[0]
+        yield o, O[0], pre_block, pre_slots, pre_pot, n_ev[0], logical[0]
 
 
-def compare(w, g, o, O, pre_block, osl, ne_o, logical_o, where):
+def compare(w, g, o, O, pre_block, osl, pre_pot, ne_o, logical_o, where):
     """One observation of one sampled sequence; returns False when the GPU
     took another valid choice inside the tie band (the trajectories part)."""
     ps = w.page_size
@@ -141,7 +171,7 @@ def compare(w, g, o, O, pre_block, osl, ne_o, logical_o, where):
     e = rel_err(g["prio"][~mism], o.prio[osl][~mism])
     assert e <= TOL_REL, (where, "prio", e)
     page_flip = np.zeros(P, bool)
-    page_flip[np.nonzero(mism)[0] // ps] = True
+    page_flip[pre_pot[np.nonzero(mism)[0]]] = True
     S_o = o.page_S[0]
     e = rel_err(g["page"][~page_flip], S_o[~page_flip])
     assert e <= TOL_REL, (where, "page", e)
@@ -156,13 +186,17 @@ def compare(w, g, o, O, pre_block, osl, ne_o, logical_o, where):
     return not mism.any()
 
 
-@pytest.mark.parametrize("config,w_attn,n_obs", [(4, 1.0, 9), (3, 1.0, 2), (4, 0.0, 3), (4, 4.0, 3)])
-def test_full_size_sampled_sequences(config, w_attn, n_obs):
+@pytest.mark.parametrize("config,w_attn,n_obs,mode", [(4, 1.0, 9, "fused"), (3, 1.0, 2, "fused"),
+                                                     (4, 0.0, 3, "fused"), (4, 4.0, 3, "fused"),
+                                                     (4, 1.0, 3, "layerwise"), (4, 1.0, 3, "aligned")])
+def test_full_size_sampled_sequences(config, w_attn, n_obs, mode):
     w = synth.make_workload(config, attn_weight=w_attn)
-    samples = (0, w.B // 2, w.B - 1) if w_attn == 1.0 else (w.B // 2,)
-    obs = gpu_run(w, n_obs, samples)
+    samples = (0, w.B // 2, w.B - 1) if (w_attn == 1.0 and mode == "fused") else (w.B // 2,)
+    obs = gpu_run(w, n_obs, samples, mode)
     for b in samples:
-        for i, (o, O, pre_block, osl, ne_o, logical_o) in enumerate(oracle_run(w, b, n_obs)):
-            if not compare(w, obs[i][b], o, O, pre_block, osl, ne_o, logical_o, (config, w_attn, b, i)):
+        runs = oracle_run(w, b, n_obs, aligned=(mode == "aligned"))
+        for i, (o, O, pre_block, osl, pre_pot, ne_o, logical_o) in enumerate(runs):
+            if not compare(w, obs[i][b], o, O, pre_block, osl, pre_pot, ne_o, logical_o,
+                           (config, w_attn, mode, b, i)):
                 break           # another valid choice inside the tie band: trajectories part here
         gc.collect()

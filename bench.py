@@ -117,7 +117,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "25"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
         except OSError:
@@ -125,19 +125,13 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.perf_counter(), line.strip()))
 
-    def stop(self):
-        if self.proc is None:
-            return None
-        self.proc.terminate()
-        try:
-            self.proc.wait(timeout=5)
-        except subprocess.TimeoutExpired:
-            self.proc.kill()
+    @staticmethod
+    def _summary(lines):
         sm, mx, reasons = [], 0.0, set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for ln in self.lines:
+        for _, ln in lines:
             parts = [x.strip() for x in ln.split(",")]
             if len(parts) < 9:
                 continue
@@ -153,6 +147,31 @@ class ClockSampler:
             return None
         return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
                 "samples": len(sm)}
+
+    def stop(self, t0: float, t1: float):
+        """Summary of the samples that arrived while the timed region ran
+        (t0..t1 on time.perf_counter, plus 50 ms for the last one).  If the
+        region was shorter than the sampling interval, the samples around it
+        are used and the result says so."""
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        return self.summarise(t0, t1)
+
+    def summarise(self, t0: float, t1: float):
+        inside = [x for x in self.lines if t0 <= x[0] <= t1 + 0.05]
+        res = self._summary(inside)
+        if res is not None:
+            res["window"] = "timed region"
+            return res
+        res = self._summary(self.lines)
+        if res is not None:
+            res["window"] = "around the timed region (shorter than the 25 ms sampling interval)"
+        return res
 
 
 # --------------------------------------------------------------- native ----
@@ -274,7 +293,7 @@ def run_native(args, rank, world, local_rank):
     wall = time.perf_counter() - wall0
     if world > 1:
         torch.distributed.barrier()
-    clk = clocks.stop() if clocks else None
+    clk = clocks.stop(wall0, wall0 + wall) if clocks else None
     prof = cache.profile_read()
     cache.profile_enable(False)
     assert cache.sync() == md.MD_OK

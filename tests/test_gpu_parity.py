@@ -13,7 +13,7 @@ if not torch.cuda.is_available():  # pragma: no cover - GPU tests only run on th
 import paper_2607_10582_gb300 as md  # noqa: E402
 import synth  # noqa: E402
 from paper_2607_10582_gb300 import build as mdbuild  # noqa: E402
-from tests.gpu_harness import Lockstep, to_dev  # noqa: E402
+from tests.gpu_harness import TOL_O_ABS, Lockstep, to_dev  # noqa: E402
 
 mdbuild.build()
 synth.build()
@@ -374,6 +374,45 @@ def test_checkpoint_carries_the_calibration_histogram():
         ls.gpu.evict(w.budget_pages)
     assert np.array_equal(res[0][0], res[1][0]) and np.array_equal(res[0][1], res[1][1])
     assert res[0][1].sum() > 0
+
+
+def test_partial_batch_leaves_the_other_sequences_untouched():
+    """Steps over sequences [0, batch) with batch < max_batch: the covered
+    sequences follow the oracle run with the same batch (outputs, evictions,
+    block tables), and the uncovered one keeps its block-table row, token
+    count and per-token state bit for bit."""
+    w = synth.custom_workload("part", L=2, Hq=16, Hkv=2, page_size=16, lengths=[800, 1300, 600],
+                              budget_frac=0.4, steps=3, seed=17, structured=True)
+    ls = Lockstep(w)
+    ls.prefill()
+    B, ps = 2, w.page_size
+    bt0 = ls.gpu.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
+    n2 = ls.gpu.query(md.MD_QUERY_TOKENS, 2)
+    slots2 = np.array([bt0[2, i // ps] * ps + i % ps for i in range(n2)])
+    state = lambda: [ls.gpu.get_state(x).cpu().numpy()[slots2] for x in
+                     (md.MD_STATE_A, md.MD_STATE_T_REF, md.MD_STATE_REGION, md.MD_STATE_WINDOW)]
+    s0 = state()
+    for t in range(1, 4):
+        q = synth.q_host(w.seed, B, w.L, w.Hq, w.Hkv, t, True)
+        kn, vn = synth.step_kv_host(w.seed, ls.pos[:B], [6] * B, w.L, w.Hkv, True)
+        out = torch.empty((B, w.L, w.Hq, 128), dtype=torch.int16, device="cuda")
+        ls.gpu.decode_step(B, to_dev(q), to_dev(kn), to_dev(vn), [6] * B, out)
+        O = ls.orc.decode_step(B, q, kn, vn, [6] * B)
+        for b in range(B):
+            ls.pos[b] += 1
+        err = float(np.max(np.abs(synth.bf16_to_f64(out.cpu().numpy().view(np.uint16)) - O)))
+        assert err <= TOL_O_ABS, (t, err)
+        st, n_ev = ls.gpu.evict(w.budget_pages[:B])
+        _, n_ev_o, _, _ = ls.orc.evict(B, w.budget_pages[:B])
+        assert list(n_ev) == list(n_ev_o), t
+        bt = ls.gpu.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
+        for b in range(B):
+            assert list(bt[b, :len(ls.orc.block[b])]) == list(ls.orc.block[b]), (t, b)
+        assert np.array_equal(bt[2], bt0[2]), t
+    assert ls.gpu.query(md.MD_QUERY_TOKENS, 2) == n2
+    for x, y in zip(state(), s0):
+        assert np.array_equal(x, y)
+    assert ls.gpu.sync() == md.MD_OK
 
 
 def test_capacity_and_argument_errors_are_synchronous():

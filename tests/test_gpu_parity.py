@@ -66,6 +66,16 @@ def test_group6_page32_structured():
     ls.check_layout()
 
 
+@pytest.mark.parametrize("Hq,Hkv,ps", [(4, 4, 16), (4, 2, 32), (2, 1, 16)])
+def test_small_gqa_groups(Hq, Hkv, ps):
+    """Groups of 1 and 2 query heads per KV head (multi-head attention at
+    G = 1): the kernel pads every group to 8 heads and masks the padding."""
+    w = synth.custom_workload(f"g{Hq // Hkv}", L=2, Hq=Hq, Hkv=Hkv, page_size=ps, lengths=[900, 2600],
+                              budget_frac=0.5, steps=6, seed=31 + Hq + Hkv, structured=True)
+    ls = Lockstep(w).run()
+    ls.check_layout()
+
+
 def test_observation_window():
     """Observation every 4 decode steps: the mass of the window's steps is
     accumulated and averaged (Sec. III-C)."""

@@ -127,7 +127,8 @@ class Lockstep:
         pre_slots = [o.slots(b) for b in range(B)]
         pre_pages = [o.page_of_token(b) for b in range(B)]
         observed = o.window_steps > 0
-        st_g, n_g = g.evict(budgets)
+        ev = torch.full((B, self.P_max), -7, dtype=torch.int32, device="cuda")
+        st_g, n_g = g.evict(budgets, ev)
         st_o, n_o, ids_o, logical_o = o.evict(B, budgets)
         assert st_g == st_o, (st_g, st_o)
         assert list(n_g) == list(n_o), (list(n_g), list(n_o))
@@ -140,6 +141,7 @@ class Lockstep:
         pscore = g.get_state(md.MD_STATE_PAGE_SCORE).cpu().numpy()
         bt = g.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
         free = g.get_state(md.MD_STATE_FREE).cpu().numpy()
+        evd = ev.cpu().numpy()
         ps = w.page_size
         fix_tref = False
         fix_blocks = False
@@ -181,12 +183,17 @@ class Lockstep:
             got = sorted(int(j) for j in np.nonzero(~np.isin(pre_block[b], bt[b, :P_pre - n_o[b]]))[0]) \
                 if n_o[b] else []
             want = logical_o[b]
+            # the evicted physical ids the call reports: the pages it evicted,
+            # in logical order, then -1
+            assert list(evd[b, n_o[b]:]) == [-1] * (self.P_max - n_o[b]), f"evicted ids padding (seq {b})"
             if got != want:
                 self._check_valid_choice(b, S_o, page_flip, got, want)
+                assert list(evd[b, :n_o[b]]) == [pre_block[b][j] for j in got], f"evicted ids (seq {b})"
                 fix_blocks = True
                 self.resyncs["evict"] += 1
             else:
                 assert list(bt[b, :len(o.block[b])]) == o.block[b], f"block table differs (seq {b})"
+                assert list(evd[b, :n_o[b]]) == list(ids_o[b]), f"evicted ids (seq {b})"
         top = len(o.free)
         if not fix_blocks:
             assert list(free[:top]) == o.free, "free stack differs"

@@ -242,6 +242,8 @@ def run_native(args, rank, world, local_rank):
         step_output = out_lm
 
     def one_step():
+        """One decode step (and the observation when the window is full);
+        returns the pages evicted per sequence, or None."""
         if args.layerwise:
             for l in range(L):
                 cache.decode_layer(l, B, q_l[l], kn_l[l], vn_l[l], regs, out_l[l])
@@ -249,7 +251,8 @@ def run_native(args, rank, world, local_rank):
             cache.decode_step(B, q, kn, vn, regs, out)
         # observation every window_k steps (k = 1 for configs 0-2 and 4)
         if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
-            cache.evict(budgets)
+            return cache.evict(budgets)[1]
+        return None
 
     if args.phase == "steady":
         one_step()
@@ -259,7 +262,8 @@ def run_native(args, rank, world, local_rank):
     if args.calib:
         cache.calib_enable(True)
     saved = cache.save_state()
-    tokens_step = sum(cache.query(md.MD_QUERY_TOKENS, b) + 1 for b in range(B))
+    tokens_saved = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+    tokens_step = sum(tokens_saved) + B
     restore = args.phase == "full"
 
     for _ in range(args.warmup):
@@ -280,16 +284,29 @@ def run_native(args, rank, world, local_rank):
     if clocks:
         clocks.start()
         time.sleep(0.3)
+    # cached tokens per sequence, tracked on the host so that the loop adds no
+    # per-sequence calls of its own: a step appends one token per sequence, an
+    # eviction removes whole pages (partly filled ones only with region-aligned
+    # pages, where the count is read back after each step instead)
+    tokens0 = tokens_saved if restore else [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+    tokens = list(tokens0)
     cache.profile_enable(True)
     wall0 = time.perf_counter()
     for i in range(args.steps):
         if restore:
             cache.load_state(saved)
-        tok_per_step.append(sum(cache.query(md.MD_QUERY_TOKENS, b) + 1 for b in range(B)))
+            tokens = list(tokens0)
+        tok_per_step.append(sum(tokens) + B)
         starts[i].record(stream)
-        one_step()
+        n_ev = one_step()
         ends[i].record(stream)
+        if args.aligned and n_ev is not None:
+            tokens = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+        else:
+            tokens = [n + 1 - (int(n_ev[b]) * ps if n_ev is not None else 0) for b, n in enumerate(tokens)]
     torch.cuda.synchronize()
+    # the host-side count agrees with the library's (checked after the timed region)
+    assert tokens == [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)], "token bookkeeping"
     wall = time.perf_counter() - wall0
     if world > 1:
         torch.distributed.barrier()

@@ -38,6 +38,8 @@ METRIC = "cached tokens scored+evicted per second per decode step"
 UNIT = "tokens/s"
 SPEC_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 10**6          # GB300 L2
+FLUSH_BYTES = 256 * 2**20       # written between timed steps when a step's K/V would fit in L2
 
 
 def parse():
@@ -265,18 +267,59 @@ def run_native(args, rank, world, local_rank):
     tokens_saved = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
     tokens_step = sum(tokens_saved) + B
     restore = args.phase == "full"
+    # a step whose K/V could stay in L2 gets the L2 flushed before it (untimed)
+    flush_buf = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev) if needs_flush(w) else None
 
-    for _ in range(args.warmup):
+    def before_step():
         if restore:
             cache.load_state(saved)
+        if flush_buf is not None:
+            flush_buf.fill_(1)
+
+    for _ in range(args.warmup):
+        before_step()
         one_step()
     torch.cuda.synchronize()
     assert cache.sync() == md.MD_OK
 
-    # ---- timed region: K steps, CUDA events on the launching stream ----
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    tok_per_step = []
+    def run_steps(profile: bool):
+        """K steps, each bracketed by CUDA events on the launching stream
+        (restore and flush happen outside the brackets).  With `profile` the
+        library also records an event pair around each of its kernels."""
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        tok_per_step = []
+        # cached tokens per sequence, tracked on the host so that the loop adds
+        # no per-sequence calls of its own: a step appends one token per
+        # sequence, an eviction removes whole pages (partly filled ones only
+        # with region-aligned pages, where the count is read back instead)
+        tokens0 = tokens_saved if restore else [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+        tokens = list(tokens0)
+        torch.cuda.synchronize()
+        cache.profile_enable(profile)
+        wall0 = time.perf_counter()
+        for i in range(args.steps):
+            before_step()
+            if restore:
+                tokens = list(tokens0)
+            tok_per_step.append(sum(tokens) + B)
+            starts[i].record(stream)
+            n_ev = one_step()
+            ends[i].record(stream)
+            if args.aligned and n_ev is not None:
+                tokens = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+            else:
+                tokens = [n + 1 - (int(n_ev[b]) * ps if n_ev is not None else 0) for b, n in enumerate(tokens)]
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+        # the host-side count agrees with the library's
+        assert tokens == [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)], "token bookkeeping"
+        prof = cache.profile_read() if profile else None
+        cache.profile_enable(False)
+        assert cache.sync() == md.MD_OK
+        return [a.elapsed_time(b) for a, b in zip(starts, ends)], tok_per_step, prof, wall0, wall
+
+    # ---- timed region: K steps, no event inside a step ----
     clocks = ClockSampler(local_rank) if not args.no_clocks else None
     if world > 1:
         torch.distributed.barrier()
@@ -284,38 +327,16 @@ def run_native(args, rank, world, local_rank):
     if clocks:
         clocks.start()
         time.sleep(0.3)
-    # cached tokens per sequence, tracked on the host so that the loop adds no
-    # per-sequence calls of its own: a step appends one token per sequence, an
-    # eviction removes whole pages (partly filled ones only with region-aligned
-    # pages, where the count is read back after each step instead)
-    tokens0 = tokens_saved if restore else [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
-    tokens = list(tokens0)
-    cache.profile_enable(True)
-    wall0 = time.perf_counter()
-    for i in range(args.steps):
-        if restore:
-            cache.load_state(saved)
-            tokens = list(tokens0)
-        tok_per_step.append(sum(tokens) + B)
-        starts[i].record(stream)
-        n_ev = one_step()
-        ends[i].record(stream)
-        if args.aligned and n_ev is not None:
-            tokens = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
-        else:
-            tokens = [n + 1 - (int(n_ev[b]) * ps if n_ev is not None else 0) for b, n in enumerate(tokens)]
-    torch.cuda.synchronize()
-    # the host-side count agrees with the library's (checked after the timed region)
-    assert tokens == [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)], "token bookkeeping"
-    wall = time.perf_counter() - wall0
+    step_ms, tok_per_step, _, wall0, wall = run_steps(False)
     if world > 1:
         torch.distributed.barrier()
     clk = clocks.stop(wall0, wall0 + wall) if clocks else None
-    prof = cache.profile_read()
-    cache.profile_enable(False)
-    assert cache.sync() == md.MD_OK
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     total_ms = float(sum(step_ms))
+
+    # ---- per-kernel times: the same K steps again with the library's event
+    # pairs around every kernel (an event between two kernels keeps them
+    # from overlapping, so these runs are not the timed ones) ----
+    _, prof_tokens, prof, _, _ = run_steps(True)
     launches = sum(n for _, n in prof.values())
     attn_ms, attn_n = prof["attention"]
 
@@ -326,8 +347,7 @@ def run_native(args, rank, world, local_rank):
         outh = torch.empty(step_output.shape, dtype=step_output.dtype).pin_memory()
         e_ms = []
         for i in range(args.warmup + args.steps):
-            if restore:
-                cache.load_state(saved)
+            before_step()
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             if args.layerwise:
@@ -349,8 +369,8 @@ def run_native(args, rank, world, local_rank):
         e2e = {"ms_per_step": float(np.mean(e_ms)), "tokens_per_step": tok_per_step[0],
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
     return dict(w=w, step_ms=step_ms, total_ms=total_ms, wall_s=wall, tokens=tok_per_step,
-                prof=prof, launches=launches, attn_ms=attn_ms, attn_n=attn_n, clocks=clk, e2e=e2e,
-                kv_bytes_per_token=L * Hkv * 2 * D * 2)
+                prof=prof, prof_tokens=prof_tokens, launches=launches, attn_ms=attn_ms, attn_n=attn_n,
+                clocks=clk, e2e=e2e, kv_bytes_per_token=L * Hkv * 2 * D * 2)
 
 
 # ------------------------------------------------------------ reference ----
@@ -459,6 +479,13 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def needs_flush(w) -> bool:
+    """Whether a step's K/V (the initial trace) is small enough to stay in L2
+    between steps, so that the L2 must be flushed before each timed step."""
+    tokens = sum(w.n0(b) + 1 for b in range(w.B))
+    return tokens * w.L * w.Hkv * 2 * w.D * 2 < 2 * L2_BYTES
+
+
 def workload_config(w, args):
     return {"workload": w.name, "batch": w.B, "tokens_per_seq": w.n0(0), "layers": w.L,
             "q_heads": w.Hq, "kv_heads": w.Hkv, "head_dim": w.D, "page_size": w.page_size,
@@ -466,7 +493,8 @@ def workload_config(w, args):
             "score_mode": "paper additive (Eq. 4)" if w.score_mode == 0 else "multiplicative",
             "phase": "full-trace step (state restored before each step)" if args.phase == "full"
             else "steady state",
-            "l2": "no flush: inputs larger than L2 (K/V read per step >> 129 MB)",
+            "l2": ("L2 flushed before every timed step (256 MiB write, untimed): a step's K/V fits in L2"
+                   if needs_flush(w) else "no flush: inputs larger than L2 (K/V read per step >> 129 MB)"),
             "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed,
             "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict",
             "calibration_histogram": bool(args.calib),
@@ -513,29 +541,35 @@ def main():
     value = all_tokens / (total_ms / 1e3)
     peak, peak_kind = peaks()
     # dominant kernel: stage-1 attention.  Algorithmic bytes per launch = the
-    # K and V rows of every cached token in every layer, plus Q and O.
-    kv_bytes = tokens * r["kv_bytes_per_token"]
+    # K and V rows of every cached token in every layer, plus Q and O; the
+    # kernel's time comes from the profiled pass over the same K steps.
     qo_bytes = 2 * w.B * w.L * w.Hq * w.D * 2
-    attn_bytes = kv_bytes + qo_bytes
+    attn_bytes = tokens * r["kv_bytes_per_token"] + qo_bytes
+    prof_tokens = float(np.mean(r["prof_tokens"]))
     launches_per_step = max(1, r["attn_n"] // args.steps)     # L with --layerwise, else 1
     attn_avg_s = r["attn_ms"] / max(1, r["attn_n"]) / 1e3
-    bytes_per_launch = attn_bytes / launches_per_step
+    bytes_per_launch = (prof_tokens * r["kv_bytes_per_token"] + qo_bytes) / launches_per_step
     achieved = bytes_per_launch / attn_avg_s / 1e9
     tpt = ncu_traffic_per_token()
-    traffic = None if tpt is None else tpt * tokens * w.L / launches_per_step
+    traffic = None if tpt is None else tpt * prof_tokens * w.L / launches_per_step
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload_config(w, args),
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": workload_config(w, args),
         "roofline": {"bound": "hbm", "kernel": "attn_mass_kernel (stage 1)", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{peak_kind} copy",
                      "traffic": traffic, "algorithmic_bytes": bytes_per_launch,
                      "launches_per_step": launches_per_step,
-                     "frac_of_8TBps_spec": achieved / SPEC_HBM_GBS},
+                     "frac_of_8TBps_spec": achieved / SPEC_HBM_GBS,
+                     "timing": "kernel time from the library's CUDA events around each launch, in a second "
+                               "pass over the same K steps right after the timed region (events between "
+                               "kernels would add gaps to the timed steps)"},
         "step_hbm_fraction": {"algorithmic_GBps": attn_bytes / (ms_per_step / 1e3) / 1e9,
                               "frac_measured": attn_bytes / (ms_per_step / 1e3) / 1e9 / peak,
                               "frac_of_8TBps_spec": attn_bytes / (ms_per_step / 1e3) / 1e9 / SPEC_HBM_GBS},
         "stage_ms_per_step": {k: v[0] / args.steps for k, v in r["prof"].items()},
+        "stage_timing": "profiled pass (see roofline.timing); stage times include the gaps the events add",
         "gpu_launches": r["launches"],
         "clocks": r["clocks"],
         "wall_s_timed": r["wall_s"],

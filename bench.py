@@ -265,7 +265,6 @@ def run_native(args, rank, world, local_rank):
         cache.calib_enable(True)
     saved = cache.save_state()
     tokens_saved = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
-    tokens_step = sum(tokens_saved) + B
     restore = args.phase == "full"
     # a step whose K/V could stay in L2 gets the L2 flushed before it (untimed)
     flush_buf = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev) if needs_flush(w) else None

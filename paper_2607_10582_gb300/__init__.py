@@ -34,6 +34,9 @@ STATUS_NAMES = {0: "MD_OK", 1: "MD_WARN_OVER_BUDGET", -1: "MD_ERR_INVALID_ARG", 
 MD_NUM_REGIONS = 7
 MD_MAX_BATCH = 256
 MD_HEAD_DIM = 128
+MD_MAX_GROUP = 8
+MD_MAX_CHUNKS = 64
+MD_MAX_CHUNK_TOKENS = 4096
 
 (MD_STATE_BLOCK_TABLE, MD_STATE_PAGE_SCORE, MD_STATE_TOKEN_PRIO, MD_STATE_A, MD_STATE_T_REF,
  MD_STATE_AHAT, MD_STATE_FREE, MD_STATE_REGION, MD_STATE_WINDOW, MD_STATE_MASS, MD_STATE_POOL,

@@ -48,11 +48,12 @@ def rel_err(g, o):
 
 
 class Lockstep:
-    def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2, layerwise=False, calib=False):
+    def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2, layerwise=False, calib=False,
+                 p_max=None):
         self.w = w
         self.layerwise = layerwise
         B = w.B
-        self.P_max = w.max_pages_per_seq()
+        self.P_max = w.max_pages_per_seq() if p_max is None else p_max
         self.P_phys = w.num_phys_pages() + phys_slack
         kw = dict(rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
                   score_mode=w.score_mode, page_reduce=w.page_reduce,

@@ -47,3 +47,22 @@ def test_c_caller_runs_a_decode_evict_loop(tmp_path):
     assert r.returncode == 0, r.stderr
     r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert r.returncode == 0 and r.stdout.strip() == "ok", (r.stdout, r.stderr)
+
+
+def test_binding_constants_match_the_header():
+    """Every limit and enumerator the Python binding mirrors has the header's
+    value (the header is the boundary's definition)."""
+    import re
+
+    import paper_2607_10582_gb300 as md
+    text = open(os.path.join(ROOT, "include", "memdecay.h")).read()
+    defines = dict(re.findall(r"#define\s+(MD_\w+)\s+(-?\d+)\b", text))
+    enums = dict(re.findall(r"\b(MD_\w+)\s*=\s*(-?\d+)\s*[,}\n/]", text))
+    values = {**enums, **defines}
+    for name in ("MD_MAX_BATCH", "MD_HEAD_DIM", "MD_MAX_GROUP", "MD_MAX_CHUNKS", "MD_MAX_CHUNK_TOKENS",
+                 "MD_CALIB_BUCKETS", "MD_CALIB_BUCKET_WIDTH", "MD_OK", "MD_ERR_DEVICE_TIMEOUT"):
+        assert name in values, name
+    mirrored = [n for n in values if hasattr(md, n)]
+    assert len(mirrored) >= 30
+    for n in mirrored:
+        assert getattr(md, n) == int(values[n]), n

@@ -466,6 +466,28 @@ def test_single_token_and_no_eviction_edges():
     ls.check_layout()
 
 
+def test_maximum_batch_of_ragged_sequences():
+    """MD_MAX_BATCH sequences in one handle, ragged from empty (the first token
+    arrives with the first decode step) to several pages with a partial last
+    page: every sequence checked at every step."""
+    lengths = [0 if i % 97 == 0 else 1 + (37 * i) % 400 for i in range(md.MD_MAX_BATCH)]
+    w = synth.custom_workload("maxbatch", L=1, Hq=8, Hkv=2, page_size=16, lengths=lengths,
+                              budget_frac=0.5, steps=3, seed=12)
+    ls = Lockstep(w).run()
+    ls.check_layout()
+
+
+def test_longest_sequence_the_chunking_allows():
+    """One sequence at the block-table limit, MD_MAX_CHUNKS chunks of
+    MD_MAX_CHUNK_TOKENS tokens (8,192 pages of 32) once the decode step's token
+    is appended, then evicted to 5% of its pages."""
+    limit = md.MD_MAX_CHUNKS * md.MD_MAX_CHUNK_TOKENS
+    w = synth.custom_workload("maxlen", L=1, Hq=8, Hkv=2, page_size=32, lengths=[limit - 1],
+                              budget_frac=0.05, steps=3, seed=13)
+    ls = Lockstep(w, p_max=limit // 32).run()
+    ls.check_layout()
+
+
 def test_device_wait_timeout_is_reported_not_hung():
     """An exchange wait that nothing completes (an injected extra arrival)
     runs out after its bounded spin; the kernel records the timeout and

@@ -277,7 +277,10 @@ md_status md_load_state(md_ctx *ctx, const void *src_dev, const void *host_blob)
  * enabled.  Stages: 0 append, 1 attention (stage 1), 2 window fold,
  * 3 score + page reduce (stages 2-3), 4 select + compact (stage 4).
  * md_profile_read synchronises the stream and returns, for each stage, the
- * summed milliseconds and the number of launches since enabling. */
+ * summed milliseconds and the number of launches since enabling.  Each event
+ * pair keeps consecutive kernels from overlapping (about 2 us per event on a
+ * GB300), so profiled steps are slower than unprofiled ones: time whole
+ * steps with profiling off. */
 md_status md_profile_enable(md_ctx *ctx, int enable);
 md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_per_stage,
                           int n_stages);

@@ -192,18 +192,21 @@ def test_calibration_histogram_and_fit():
     Lockstep(w3, calib=True).run().check_calibration()
 
 
-def test_config1_first_steps():
-    """Config 1 geometry (Qwen2.5-1.5B, 28 layers, 12/2 heads), 1,700 tokens."""
+def test_config1_full_run():
+    """Config 1 end to end (Qwen2.5-1.5B geometry, 28 layers, 12/2 heads):
+    1,700-token trace, all 256 decode steps, eviction to 25% of the pages."""
     ls = Lockstep(synth.make_workload(1))
-    ls.run(steps=20)
+    ls.run()
     ls.check_layout()
 
 
 def test_config2_first_steps():
     """Config 2 geometry (Qwen2.5-3B, 36 layers, 16/2), 32 sequences with
-    Dirichlet region spans and insertion offsets."""
+    Dirichlet region spans and insertion offsets: the full-trace step and 31
+    steady steps, every sequence at every step (two page boundaries pass, so
+    appends take pages the evictions freed)."""
     ls = Lockstep(synth.make_workload(2))
-    ls.run(steps=3)
+    ls.run(steps=32)
     ls.check_layout()
 
 

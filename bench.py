@@ -21,6 +21,7 @@ from __future__ import annotations
 
 import argparse
 import copy
+import ctypes
 import hashlib
 import json
 import os
@@ -58,6 +59,8 @@ def parse():
                     help="decode through md_decode_layer, one call per layer")
     ap.add_argument("--aligned", action="store_true",
                     help="region-aligned page allocation (a fresh page at each region boundary)")
+    ap.add_argument("--structured", action="store_true",
+                    help="keys and queries with region structure and hot tokens (refreshes fire)")
     ap.add_argument("--calib", action="store_true",
                     help="gather the calibration histogram (Eqs. 6-7) during observation steps")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -202,7 +205,7 @@ def run_native(args, rank, world, local_rank):
     for r in range(7):
         cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
     lib = synth.lib()
-    kap = None
+    kap = (ctypes.c_float * 9)(*synth.KAPPA_STRUCT) if w.structured else None
     nmax = max(w.n0(b) for b in range(B))
     kbuf = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
     vbuf = torch.empty_like(kbuf)
@@ -396,6 +399,8 @@ def oracle_sample(w, layers: int, seq: int = 0):
 def make_workload(args, seed):
     import synth
     over = {"attn_weight": args.w} if args.config == 4 else {}
+    if args.structured:
+        over["structured"] = True
     w = synth.make_workload(args.config, seed=seed, **over)
     if args.max_tokens:
         n = args.max_tokens
@@ -497,7 +502,9 @@ def workload_config(w, args):
             "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed,
             "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict",
             "calibration_histogram": bool(args.calib),
-            "page_allocation": "region-aligned" if args.aligned else "contiguous"}
+            "page_allocation": "region-aligned" if args.aligned else "contiguous",
+            "values": ("structured: per-region key offsets along one direction, 2% hot keys (Fig. 3 mass ratios)"
+                       if w.structured else "iid N(0,1)")}
 
 
 def combine_over_ranks(total_ms: float, tokens_total: float, device):

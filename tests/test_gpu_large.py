@@ -2,8 +2,9 @@
 configuration (the whole batch, 77 GB of K/V per step, on the GPU), checked
 on sampled sequences {0, B/2, B-1} that the oracle recomputes one by one: at
 the full-trace observation and at the steady observations after it.  Config 4
-is also run through the layer-by-layer entry point and with region-aligned
-pages (pages then hold different numbers of tokens).
+is also run through the layer-by-layer entry point, with region-aligned
+pages (pages then hold different numbers of tokens) and with structured keys
+(refreshes fire).
 
 Sequences are independent in every stage except the shared page pool, so the
 oracle runs a sampled sequence alone (its physical page ids differ) and the
@@ -57,12 +58,14 @@ def gpu_run(w, n_obs, samples, mode="fused"):
     for r in range(7):
         cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
     lib = synth.lib()
+    sflag = int(w.structured)
+    kap = (synth.ctypes.c_float * 9)(*synth.KAPPA_STRUCT) if w.structured else None
     nmax = max(w.n0(b) for b in range(B))
     kb = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
     vb = torch.empty_like(kb)
     for b in range(B):
         rd = torch.from_numpy(w.regions[b]).to(dev)
-        assert lib.synth_fill_kv_dev(w.seed, 0, None, b, L, Hkv, D, 0, w.n0(b), rd.data_ptr(),
+        assert lib.synth_fill_kv_dev(w.seed, sflag, kap, b, L, Hkv, D, 0, w.n0(b), rd.data_ptr(),
                                      kb.data_ptr(), vb.data_ptr(), None) == 0
         cache.append_tokens(b, w.regions[b], kb.data_ptr(), vb.data_ptr(), w.insert_steps[b])
         torch.cuda.synchronize()
@@ -79,8 +82,8 @@ def gpu_run(w, n_obs, samples, mode="fused"):
         for k in range(w.window_k):
             t += 1
             pos = torch.tensor([w.n0(b) + t - 1 for b in range(B)], dtype=torch.int32, device=dev)
-            assert lib.synth_fill_q_dev(w.seed, 0, None, B, L, Hq, Hq // Hkv, D, t, q.data_ptr(), None) == 0
-            assert lib.synth_fill_step_kv_dev(w.seed, 0, None, B, L, Hkv, D, pos.data_ptr(), rdev.data_ptr(),
+            assert lib.synth_fill_q_dev(w.seed, sflag, kap, B, L, Hq, Hq // Hkv, D, t, q.data_ptr(), None) == 0
+            assert lib.synth_fill_step_kv_dev(w.seed, sflag, kap, B, L, Hkv, D, pos.data_ptr(), rdev.data_ptr(),
                                               kn.data_ptr(), vn.data_ptr(), None) == 0
             if mode == "layerwise":
                 # a model hands each layer its own contiguous [B][heads][D] tensors
@@ -136,15 +139,16 @@ def oracle_run(w, b, n_obs, aligned=False):
     o = om.Oracle(cfg)
     for r in range(7):
         o.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
-    k, v = synth.kv_host(w.seed, b, w.L, w.Hkv, 0, n, w.regions[b])
+    k, v = synth.kv_host(w.seed, b, w.L, w.Hkv, 0, n, w.regions[b], w.structured)
     o.append_tokens(0, w.regions[b], k, v, w.insert_steps[b])
     del k, v
     t = 0
     for _ in range(n_obs):
         for _k in range(w.window_k):
             t += 1
-            q = synth.q_host(w.seed, w.B, w.L, w.Hq, w.Hkv, t)[b:b + 1]
-            kn, vn = synth.kv_host(w.seed, b, w.L, w.Hkv, n + t - 1, 1, np.array([w.decode_region], np.uint8))
+            q = synth.q_host(w.seed, w.B, w.L, w.Hq, w.Hkv, t, w.structured)[b:b + 1]
+            kn, vn = synth.kv_host(w.seed, b, w.L, w.Hkv, n + t - 1, 1, np.array([w.decode_region], np.uint8),
+                                   w.structured)
             O = o.decode_step(1, q, kn[:, :, 0, :][None], vn[:, :, 0, :][None], [w.decode_region])
         pre_block = list(o.block[0])
         pre_slots = o.slots(0)
@@ -188,15 +192,20 @@ def compare(w, g, o, O, pre_block, osl, pre_pot, ne_o, logical_o, where):
 
 @pytest.mark.parametrize("config,w_attn,n_obs,mode", [(4, 1.0, 9, "fused"), (3, 1.0, 2, "fused"),
                                                      (4, 0.0, 3, "fused"), (4, 4.0, 3, "fused"),
-                                                     (4, 1.0, 3, "layerwise"), (4, 1.0, 3, "aligned")])
+                                                     (4, 1.0, 3, "layerwise"), (4, 1.0, 3, "aligned"),
+                                                     (4, 1.0, 3, "structured")])
 def test_full_size_sampled_sequences(config, w_attn, n_obs, mode):
-    w = synth.make_workload(config, attn_weight=w_attn)
+    w = synth.make_workload(config, attn_weight=w_attn, structured=(mode == "structured"))
     samples = (0, w.B // 2, w.B - 1) if (w_attn == 1.0 and mode == "fused") else (w.B // 2,)
     obs = gpu_run(w, n_obs, samples, mode)
+    refreshed = 0
     for b in samples:
         runs = oracle_run(w, b, n_obs, aligned=(mode == "aligned"))
         for i, (o, O, pre_block, osl, pre_pot, ne_o, logical_o) in enumerate(runs):
+            refreshed += int(np.count_nonzero((o.t_ref[osl] == o.t) & (o.t_ins[osl] < o.t)))
             if not compare(w, obs[i][b], o, O, pre_block, osl, pre_pot, ne_o, logical_o,
                            (config, w_attn, mode, b, i)):
                 break           # another valid choice inside the tie band: trajectories part here
         gc.collect()
+    if mode == "structured":
+        assert refreshed > 0   # the structured keys make Eq. 3's refresh fire

@@ -210,6 +210,17 @@ def test_config2_first_steps():
     ls.check_layout()
 
 
+def test_config2_structured():
+    """Config 2 with structured keys and queries (per-region offsets, hot
+    tokens): refreshes fire, every sequence checked at every step."""
+    ls = Lockstep(synth.make_workload(2, structured=True))
+    ls.run(steps=12)
+    ls.check_layout()
+    o = ls.orc
+    sl = np.concatenate([o.slots(b) for b in range(ls.w.B)])
+    assert np.count_nonzero((o.t_ref[sl] == o.t) & (o.t_ins[sl] < o.t)) > 0   # refreshed, not new
+
+
 def _small_run(seed):
     w = synth.custom_workload("det", L=2, Hq=16, Hkv=2, page_size=16, lengths=[700, 1500],
                               budget_frac=0.5, steps=6, seed=seed, structured=True)

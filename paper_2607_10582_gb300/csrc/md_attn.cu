@@ -4,8 +4,8 @@
  *
  * Work unit: (sequence b, layer l, KV head kvh, chunk j of the sequence's
  * pages).  The chunks of one (b, l, kvh) item split its pages (flash-decoding
- * style) so that ~all 152 SMs stream K/V at once.  One persistent cooperative
- * CTA per SM walks the units c, c+grid, c+2*grid, ...
+ * style) so that ~all 152 SMs stream K/V at once.  Two persistent cooperative
+ * CTAs per SM; CTA c walks the units c, c+grid, c+2*grid, ...
  *
  * Per CTA: warp 0 is the producer.  One elected lane issues, per page, two
  * TMA tile loads (cp.async.bulk.tensor, 128-byte swizzle, L2 evict_first) of
@@ -28,11 +28,11 @@
  * combines the partials (its slice of the output O) and turns the stored
  * scores into masses, one fp32 row per (layer, KV head) indexed by physical
  * slot.  Raw scores live in two slots per CTA; the consumers reuse a slot only
- * after the finisher has released it (mbarrier hand-off both ways), so the
- * finish never stalls the copy stream.  All waits are bounded; on expiry the kernel
- * records MD_ERR_DEVICE_TIMEOUT, raises an abort flag every CTA polls, drains
- * its in-flight copies and returns.  No float atomics: results are
- * bit-identical run to run. */
+ * after the finisher has released it (mbarrier hand-off both ways), so a
+ * unit's finish overlaps the streaming of the next one.  All waits are
+ * bounded; on expiry the kernel records MD_ERR_DEVICE_TIMEOUT, raises an abort
+ * flag every CTA polls, drains its in-flight copies and returns.  No float
+ * atomics: results are bit-identical run to run. */
 #include <cuda_bf16.h>
 #include <float.h>
 
@@ -477,7 +477,7 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       mbar_init(smem_u32(&fdone[s]), 1);
     }
     mbar_init(smem_u32(&mdone[0]), 1);
-    flag[0] = flag[1] = flag[2] = flag[3] = 0;
+    flag[0] = flag[1] = flag[2] = 0;
     fence_barrier_init();
   }
   __syncthreads();

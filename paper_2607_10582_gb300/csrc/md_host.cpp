@@ -259,18 +259,22 @@ md_status launch_fold(md_ctx *c) {
  *
  * A split of every sequence into C chunks, with G a multiple of C and the
  * unit count a multiple of G, has no such boundary and gives every CTA the
- * same work.  Among those with G >= 0.84 glim (fewer CTAs would no longer
- * keep HBM saturated) the one with the largest G, then the fewest units, is
- * taken when its streamed pages plus per-unit overheads are below the plain
- * split's, counted with a penalty of 0.4 / rounds when the plain split has
- * such boundaries (fitted to the measurement above).  Returns the plain
- * split (G = 0) otherwise. */
+ * same work, where the plain split's last round may be partly empty.  Costs
+ * are CTA-time in pages (HBM is shared, so the time of a launch that keeps
+ * it saturated follows the CTAs' summed busy time): the aligned split's
+ * streamed pages plus per-unit overheads, against the plain split's makespan
+ * times its grid, with a penalty of 0.4 / rounds when its rounds end inside
+ * items (fitted to the measurement above).  Among aligned splits with
+ * G >= 0.84 glim (fewer CTAs would not keep HBM saturated) the largest G,
+ * then the fewest units, is taken when cheaper.  A plain split of one round
+ * is kept: such a launch is too short to be HBM-bound and its time is the
+ * largest unit's.  Returns the plain split (G = 0) otherwise. */
 struct Aligned {
   int T, G;
 };
 
-Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0, long long glim,
-                         double ov, double l2_budget) {
+Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0, double makespan0,
+                         long long glim, double ov, double l2_budget) {
   const int ps = c->cfg.page_size;
   const int cmax = c->lay.chunk_stride;
   const int max_chunk_pages = std::max(1, c->lay.scratch_tokens / ps);
@@ -292,20 +296,21 @@ Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0
   if (U0 == 0 || active == 0) return {T0, 0};
   const long long G0 = std::max(1LL, std::min(U0, glim));
   const long long rounds = (U0 + G0 - 1) / G0;
+  if (rounds < 2) return {T0, 0};
   int inside = 0;
   for (long long k = 1, b = 0; k < rounds; ++k) {
     const long long x = k * G0;
     while (start[b + 1] <= x) ++b;
     if ((x - start[b]) % ch[b] != 0) ++inside;
   }
-  double cost0 = pages + ov * (double)U0;
+  double cost0 = makespan0 * (double)G0;
   if (inside > 0) cost0 *= 1.0 + 0.4 / (double)rounds;
   /* aligned splits */
   const long long itot = (long long)active * items;
   Aligned best{T0, 0};
   long long bestG = 0;
   double bestCost = cost0;
-  for (int C = 2; C <= cmax; ++C) {
+  for (int C = 1; C <= cmax; ++C) {
     const int T = (Pmax + C - 1) / C;
     if (T > max_chunk_pages) continue;
     bool uniform = true;
@@ -416,7 +421,7 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
   }
   if (bestT == 0) bestT = max_chunk_pages;
   if (!same && c->force_chunks == 0 && c->grid_cap == 0) {
-    const Aligned a = aligned_schedule(c, batch, items, Pmax, bestT, glim, ov, l2_budget);
+    const Aligned a = aligned_schedule(c, batch, items, Pmax, bestT, best, glim, ov, l2_budget);
     bestT = a.T;
     bestG = a.G;
   }

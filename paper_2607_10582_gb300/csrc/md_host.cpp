@@ -343,7 +343,8 @@ Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0
  * difference array gives all CTA loads in O(batch + G).  A unit costs its
  * pages plus a fixed per-unit overhead (Q load, merge, publish, ramp),
  * expressed as K/V bytes streamed.  At most MD_MAX_CHUNK_TOKENS tokens per
- * chunk; the live raw-score scratch must stay inside L2. */
+ * chunk; the live raw-score scratch must stay inside L2.  A round-aligned
+ * schedule (aligned_schedule) may then replace the split and the grid. */
 void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid) {
   const int ps = c->cfg.page_size;
   const int items = layers * c->cfg.num_kv_heads;

@@ -124,7 +124,9 @@ size_t md_workspace_size(const md_config *cfg);
 
 /* Validates cfg, lays out the workspace, and enqueues its initialisation
  * (empty cache, free stack [P-1, ..., 0] so the first page taken is 0).
- * Region parameters start as b = 0, half-life = +inf, not pinned. */
+ * Region parameters start as b = 0, half-life = +inf, not pinned.
+ * MD_ERR_CAPACITY if the device holds fewer than MD_MAX_CHUNKS attention CTAs
+ * at once (every chunk of an item must fit in one round of the grid). */
 md_status md_create(const md_config *cfg, md_ctx **out);
 
 /* Structural prior of one region (Sec. III-B, Table 1): base priority
@@ -291,7 +293,9 @@ md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_p
  *                             on its next launch (a wait nothing completes;
  *                             the kernel then reports MD_ERR_DEVICE_TIMEOUT)
  *   MD_DEBUG_GRID_LIMIT       cap on the attention kernel's persistent CTAs
- *                             (0 = all that fit on the device)
+ *                             (0 = all that fit on the device; otherwise at
+ *                             least MD_MAX_CHUNKS, so that all chunks of an
+ *                             item fit in one round of the grid)
  *   MD_DEBUG_UNIT_OVERHEAD    per-unit cost, in KiB of K/V streamed, that the
  *                             attention work planner adds to each chunk
  *                             (default 112; 0..65536)

@@ -552,6 +552,10 @@ MD_API md_status md_create(const md_config *cfg, md_ctx **out) {
     delete c;
     return MD_ERR_CUDA;
   }
+  if (c->grid_limit < MD_MAX_CHUNKS) {   // an item's chunks must fit in one round
+    delete c;
+    return MD_ERR_CAPACITY;
+  }
   /* TMA descriptor over the pool viewed as [rows][128] bf16, rows = (layer,
    * page, KV head, K|V, token); one box = one page's K and V rows x 64 dims,
    * 128-byte swizzled. */
@@ -1319,7 +1323,10 @@ MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
     return MD_OK;
   }
   if (key == MD_DEBUG_GRID_LIMIT) {
-    if (value < 0) return fail(c, MD_ERR_INVALID_ARG, "negative grid limit");
+    /* all chunks of an item must fit in one round of the grid (the order
+     * that keeps the kernel's cross-CTA waits free of cycles) */
+    if (value < 0 || (value > 0 && value < MD_MAX_CHUNKS))
+      return fail(c, MD_ERR_INVALID_ARG, "grid limit must be 0 or at least MD_MAX_CHUNKS");
     c->grid_cap = (int)std::min<int64_t>(value, MAX_GRID);
     return MD_OK;
   }

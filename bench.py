@@ -12,6 +12,11 @@ w = 1), at its full-trace step: the first decode step after the prefill,
 attending over the whole trace (77 GB of K/V) and evicting down to budget.
 The device state is restored (untimed) before every timed step, so every
 step does that full work; `--phase steady` times continuing steps instead.
+Each timed step is bracketed by CUDA events on the launching stream and holds
+no other event; the per-kernel times behind the roofline come from a second
+pass over the same steps with the library's event pairs.  Where a step's K/V
+would fit in L2 (configs 0 and 1), a 256 MiB write flushes it before each
+step, outside the brackets.
 
 `--impl reference` times the fp64 CPU oracle on the host cores on a bounded
 sample of the same workload (the paper ships no code; the oracle is the

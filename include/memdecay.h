@@ -372,14 +372,24 @@ md_status md_calib_fit(const double *mass_sum, const int64_t *count, int n_bucke
  *   stream           cudaStream_t
  *
  * Limits: the work must fit the 24 MiB array.  Each (sequence, layer, KV
- * head) is split into chunks of at most 1,024 tokens, and the partials of all
- * of them must fit next to the score rows.  Larger work (for instance very
- * long sequences times many layers and sequences) is rejected with
- * MD_ERR_CAPACITY before anything is launched; bad arguments with
- * MD_ERR_INVALID_ARG.
+ * head) is split into C chunks of at most 1,024 tokens (C <= MD_MAX_CHUNKS),
+ * as few as keep every CTA of the grid busy.  The array holds one arrival
+ * counter per item, two rows of chunk scores (32 bytes per token) per CTA of
+ * the launched grid, and, when C > 1, C partials of 4,352 bytes per item.
+ * In practice: any batch whose sequences all hold at most 1,024 tokens (one
+ * chunk per item, no partials) fits; so does, for instance, 16 sequences of
+ * 3,000 tokens over 16 layers and 2 KV heads (C = 4, about 23.5 MiB).  Work
+ * that fits no split (for instance 32 sequences of 1,700 tokens over 36
+ * layers and 2 KV heads) is rejected with MD_ERR_CAPACITY before anything is
+ * launched, and so is a split whose C exceeds the CTAs the device holds at
+ * once (all chunks of an item must run in one round of the persistent
+ * grid); bad arguments with MD_ERR_INVALID_ARG.
  *
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress), so make that first call before any stream capture.
+ * The first call on a device, with that device current, looks up the
+ * array's device address (cudaGetSymbolAddress), the kernel's resident CTAs
+ * (occupancy query; it also sets the kernel's shared-memory limit) and the
+ * driver's tensor-map encoder, and keeps them for the process; make that
+ * first call before any stream capture.
  * Every call on a device shares the same array and clears its counters and
  * status words on the stream before the kernel; calls whose GPU work overlaps
  * (other streams, other threads) race on the array and must be serialised by

@@ -853,7 +853,7 @@ cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &tmap, int g
 namespace md {
 
 constexpr size_t NOALLOC_BYTES = (size_t)24 << 20;     // 24 MiB, every device that loads us
-constexpr int NOALLOC_TOKENS = 1024;                   // scratch rows per CTA slot
+constexpr int NOALLOC_TOKENS = 1024;                   // tokens per chunk at most
 constexpr size_t NOALLOC_STATUS_BYTES = 256;
 
 static __device__ __align__(256) uint8_t g_noalloc_scratch[NOALLOC_BYTES];
@@ -867,24 +867,94 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[NOALLOC_BYTES];
 
 namespace {
 
-/* Device address of g_noalloc_scratch, looked up once per device. */
-std::mutex g_noalloc_mu;
-void *g_noalloc_addr[128] = {nullptr};
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-cudaError_t noalloc_base(void **out) {
+/* What a call needs from its device, found by the first call on that device
+ * (with the device current) and kept for the process: the device address of
+ * g_noalloc_scratch and the attention CTAs resident at once, for pages of 16
+ * and of 32 tokens (the latter also sets the kernel's shared-memory limit). */
+struct NoallocDevice {
+  void *base = nullptr;
+  int grid_limit[2] = {0, 0};
+};
+constexpr int NOALLOC_MAX_DEVICES = 128;
+std::mutex g_noalloc_mu;
+NoallocDevice g_noalloc_dev[NOALLOC_MAX_DEVICES];
+EncodeTiledFn g_encode = nullptr;
+
+cudaError_t noalloc_device(int ps, void **base, int *grid_limit, EncodeTiledFn *encode) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 128) return cudaErrorInvalidDevice;
+  if (dev < 0 || dev >= NOALLOC_MAX_DEVICES) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
+  NoallocDevice &d = g_noalloc_dev[dev];
+  if (!d.base) {
     void *p = nullptr;
     e = cudaGetSymbolAddress(&p, md::g_noalloc_scratch);
     if (e != cudaSuccess) return e;
-    g_noalloc_addr[dev] = p;
+    d.base = p;
   }
-  *out = g_noalloc_addr[dev];
+  int &gl = d.grid_limit[ps == 32 ? 1 : 0];
+  if (gl <= 0) {
+    gl = md::attention_grid_limit(ps);
+    if (gl <= 0) return cudaErrorUnknown;
+  }
+  if (!g_encode) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorUnknown;
+    g_encode = (EncodeTiledFn)fn;
+  }
+  *base = d.base;
+  *grid_limit = gl;
+  *encode = g_encode;
   return cudaSuccess;
+}
+
+/* One candidate split of every (sequence, layer, KV head) item into C chunks
+ * and the bytes of the fixed array it occupies: status words, one arrival
+ * counter per item, two score rows of the chunk's tokens per CTA of the grid
+ * that will be launched, and (only when some item has several chunks) C
+ * partials per item. */
+struct NoallocPlan {
+  int C, T, grid, scratch_tokens;
+  long long units;
+  size_t counters_bytes, scores_bytes, partial_bytes;
+};
+
+NoallocPlan noalloc_plan(int C, int Pmax, int ps, const int *n_pages, int batch, long long items_per_seq,
+                         int grid_limit) {
+  NoallocPlan pl;
+  pl.C = C;
+  pl.T = (Pmax + C - 1) / C;
+  pl.scratch_tokens = (pl.T * ps + 15) / 16 * 16;
+  pl.units = 0;
+  bool multi = false;
+  for (int b = 0; b < batch; ++b) {
+    int ch = (n_pages[b] + pl.T - 1) / pl.T;
+    if (ch > C) ch = C;
+    if (ch > n_pages[b]) ch = n_pages[b];
+    multi |= ch > 1;
+    pl.units += items_per_seq * ch;
+  }
+  pl.grid = (int)(pl.units < grid_limit ? pl.units : grid_limit);
+  if (pl.grid < 1) pl.grid = 1;
+  const long long items = items_per_seq * batch;
+  pl.counters_bytes = (size_t)((items * 4 + 255) / 256 * 256);
+  pl.scores_bytes = (size_t)pl.grid * 2 * pl.scratch_tokens * md::GP * 4;
+  pl.partial_bytes = multi ? (size_t)items * C * md::PARTIAL_FLOATS * 4 : 0;
+  return pl;
+}
+
+bool noalloc_fits(const NoallocPlan &pl) {
+  return md::NOALLOC_STATUS_BYTES + pl.counters_bytes + pl.scores_bytes + pl.partial_bytes <=
+         md::NOALLOC_BYTES;
 }
 
 }  // namespace
@@ -910,18 +980,11 @@ extern "C" __attribute__((visibility("default"))) md_status md_attend_mass_noall
     if (n_tokens_host[b] < 1 || (long long)n_tokens_host[b] > (long long)max_pages_per_seq * ps)
       return MD_ERR_INVALID_ARG;
 
-  /* plan: chunks of at most NOALLOC_TOKENS tokens, partials for every chunk
-   * of every item, all inside the fixed array */
-  const long long items = (long long)batch * num_layers * num_kv_heads;
-  int grid_limit = attention_grid_limit(ps);
-  if (grid_limit <= 0) return MD_ERR_CUDA;
-  const size_t scores_bytes = (size_t)grid_limit * 2 * NOALLOC_TOKENS * GP * 4;
-  const size_t counters_bytes = (size_t)((items * 4 + 255) / 256 * 256);
-  if (NOALLOC_STATUS_BYTES + counters_bytes + scores_bytes >= NOALLOC_BYTES) return MD_ERR_CAPACITY;
-  const size_t part_room = NOALLOC_BYTES - NOALLOC_STATUS_BYTES - counters_bytes - scores_bytes;
-  long long cstride = (long long)(part_room / ((size_t)items * PARTIAL_FLOATS * 4));
-  if (cstride > MD_MAX_CHUNKS) cstride = MD_MAX_CHUNKS;
-  const int cap_pages = NOALLOC_TOKENS / ps;
+  void *base = nullptr;
+  int grid_limit = 0;
+  EncodeTiledFn encode = nullptr;
+  if (noalloc_device(ps, &base, &grid_limit, &encode) != cudaSuccess) return MD_ERR_CUDA;
+
   AttnParams ap;
   memset(&ap, 0, sizeof(ap));
   int Pmax = 1;
@@ -931,35 +994,42 @@ extern "C" __attribute__((visibility("default"))) md_status md_attend_mass_noall
     ap.n_tokens[b] = n_tokens_host[b];
     if (P > Pmax) Pmax = P;
   }
-  /* the smallest chunk count that fits the per-chunk cap, then more chunks
-   * while the grid is not yet full and they fit the partials room */
-  int need = (Pmax + cap_pages - 1) / cap_pages;
-  if (need > cstride) return MD_ERR_CAPACITY;
-  int C = need;
-  while (C < cstride && C < Pmax && items * C < grid_limit) ++C;
-  const int T = (Pmax + C - 1) / C;
+  /* the split: chunks of at most NOALLOC_TOKENS tokens and at most
+   * MD_MAX_CHUNKS per item, as few as fill the grid, among those that fit
+   * the fixed array (the most that fit if none fills it).  Every chunk of an
+   * item must fit in one round of the grid (a finisher waits only for chunks
+   * placed before its own next unit), so C may not exceed the grid. */
+  const long long items_per_seq = (long long)num_layers * num_kv_heads;
+  const int cap_pages = NOALLOC_TOKENS / ps;
+  const int need = (Pmax + cap_pages - 1) / cap_pages;
+  const int cmax = Pmax < MD_MAX_CHUNKS ? Pmax : MD_MAX_CHUNKS;
+  NoallocPlan best;
+  best.C = 0;
+  for (int C = need; C <= cmax; ++C) {
+    const NoallocPlan pl = noalloc_plan(C, Pmax, ps, ap.n_pages, batch, items_per_seq, grid_limit);
+    if (C > pl.grid || !noalloc_fits(pl)) continue;
+    best = pl;
+    if (pl.units >= grid_limit) break;
+  }
+  if (best.C == 0) return MD_ERR_CAPACITY;
   long long U = 0;
   for (int b = 0; b < batch; ++b) {
-    const int P = ap.n_pages[b];
-    int ch = (P + T - 1) / T;
-    if (ch > C) ch = C;
-    if (ch > P) ch = P;
+    int ch = (ap.n_pages[b] + best.T - 1) / best.T;
+    if (ch > best.C) ch = best.C;
+    if (ch > ap.n_pages[b]) ch = ap.n_pages[b];
     ap.chunks[b] = ch;
     ap.unit_start[b] = (int)U;
-    U += (long long)num_layers * num_kv_heads * ch;
+    U += items_per_seq * ch;
   }
   ap.unit_start[batch] = (int)U;
   ap.total_units = (int)U;
   ap.n_seqs = batch;
 
-  void *base = nullptr;
-  cudaError_t e = noalloc_base(&base);
-  if (e != cudaSuccess) return MD_ERR_CUDA;
   uint8_t *s8 = (uint8_t *)base;
   ap.status = (int *)s8;
   ap.counters = (int *)(s8 + NOALLOC_STATUS_BYTES);
-  ap.scratch = (float *)(s8 + NOALLOC_STATUS_BYTES + counters_bytes);
-  ap.partials = (float *)(s8 + NOALLOC_STATUS_BYTES + counters_bytes + scores_bytes);
+  ap.scratch = (float *)(s8 + NOALLOC_STATUS_BYTES + best.counters_bytes);
+  ap.partials = (float *)(s8 + NOALLOC_STATUS_BYTES + best.counters_bytes + best.scores_bytes);
   ap.q = (const uint16_t *)q_dev;
   ap.out = (uint16_t *)out_dev;
   ap.block_table = block_table_dev;
@@ -975,39 +1045,27 @@ extern "C" __attribute__((visibility("default"))) md_status md_attend_mass_noall
   ap.P_phys = num_phys_pages;
   ap.P_max = max_pages_per_seq;
   ap.slots = (long long)num_phys_pages * ps;
-  ap.scratch_tokens = NOALLOC_TOKENS;
-  ap.chunk_stride = (int)cstride;
+  ap.scratch_tokens = best.scratch_tokens;
+  ap.chunk_stride = best.C;
   ap.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
   ap.spin_limit_ns = 2000000000LL;
   ap.extra_arrivals = 0;
 
-  void *fn = nullptr;
-  cudaDriverEntryPointQueryResult qres;
-  e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
-                                       &qres);
-  if (e != cudaSuccess || qres != cudaDriverEntryPointSuccess || !fn) return MD_ERR_CUDA;
-  typedef CUresult (*EncodeFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
-                               const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
-                               const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
-                               CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
   CUtensorMap tmap;
   cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)D * 2};
   cuuint32_t box[2] = {64, (cuuint32_t)(2 * ps)};
   cuuint32_t estr[2] = {1, 1};
-  if (((EncodeFn)fn)(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void *)kv_pool_dev, dims,
-                     strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+  if (encode(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void *)kv_pool_dev, dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return MD_ERR_INVALID_ARG;
 
   /* the array keeps the previous call's contents: counters and status words
    * must start at zero */
   cudaStream_t st = (cudaStream_t)stream;
-  e = cudaMemsetAsync(s8, 0, NOALLOC_STATUS_BYTES + counters_bytes, st);
+  cudaError_t e = cudaMemsetAsync(s8, 0, NOALLOC_STATUS_BYTES + best.counters_bytes, st);
   if (e != cudaSuccess) return MD_ERR_CUDA;
-  int grid = (int)(U < grid_limit ? U : grid_limit);
-  if (grid < 1) grid = 1;
-  e = launch_attention(ap, tmap, grid, st);
+  e = launch_attention(ap, tmap, best.grid, st);
   return e == cudaSuccess ? MD_OK : MD_ERR_CUDA;
 }

@@ -24,9 +24,19 @@ mdbuild.build()
 synth.build()
 
 
-@pytest.mark.parametrize("Hq,ps,lengths", [(16, 16, [900, 2500]), (12, 32, [3000, 70, 1500])])
-def test_noalloc_matches_workspace_path_twice(Hq, ps, lengths):
-    w = synth.custom_workload("noalloc", L=2, Hq=Hq, Hkv=2, page_size=ps, lengths=lengths,
+@pytest.mark.parametrize("L,Hq,ps,lengths", [
+    (2, 16, 16, [900, 2500]),
+    (2, 12, 32, [3000, 70, 1500]),
+    # many items and long sequences: the split that fills the grid (3 chunks
+    # per item) does not fit the fixed array, so the call takes 4; the
+    # 40-token sequence gets fewer chunks than the others
+    (16, 16, 16, [3000] * 7 + [40] + [3000] * 8),
+    # a serving batch shaped like the 3B geometry at budget: one chunk per
+    # item, no partials
+    (36, 16, 16, [420 + 9 * i for i in range(32)]),
+])
+def test_noalloc_matches_workspace_path_twice(L, Hq, ps, lengths):
+    w = synth.custom_workload("noalloc", L=L, Hq=Hq, Hkv=2, page_size=ps, lengths=lengths,
                               budget_frac=0.5, steps=4, seed=21, structured=True)
     B, L, Hkv, D = w.B, w.L, w.Hkv, 128
     c = md.Cache(L, Hq, Hkv, ps, B, w.max_pages_per_seq(), w.num_phys_pages())
@@ -73,6 +83,11 @@ def test_noalloc_rejects_work_beyond_its_fixed_scratch():
     n_tok = np.full(256, 4096, np.int32)
     p = dummy.data_ptr()
     st = md.lib().md_attend_mass_noalloc(p, p, n_tok.ctypes.data, p, p, p, 256, 36, 16, 2, 16, 4096, 64, None)
+    assert st == md.MD_ERR_CAPACITY
+    # the 3B geometry's full trace, 32 x 1,700 tokens: two chunks per item
+    # would need about 37 MiB of scores and partials
+    n_tok2 = np.full(32, 1700, np.int32)
+    st = md.lib().md_attend_mass_noalloc(p, p, n_tok2.ctypes.data, p, p, p, 32, 36, 16, 2, 16, 107, 64, None)
     assert st == md.MD_ERR_CAPACITY
     st = md.lib().md_attend_mass_noalloc(p, p, n_tok.ctypes.data, p, p, p, 1, 2, 16, 2, 24, 4096, 64, None)
     assert st == md.MD_ERR_INVALID_ARG

@@ -31,6 +31,79 @@ TOL_FLOOR = 1e-30
 TIE_REL = 1e-5
 
 
+class TieStats:
+    """How often the tie band decided anything.
+
+    Per observation and sequence with an eviction: the relative gap between
+    the selection boundary (the largest oracle page score S among the evicted
+    pages) and the smallest score among the kept evictable pages.  A gap
+    within TIE_REL means the oracle's own decision sat inside the band, where
+    the GPU could take another valid choice.  For every choice the GPU took
+    differently (an adoption), the distance of the swapped pages from the
+    boundary, relative to it: the largest such distance is the narrowest band
+    under which the run would still have passed.  Refresh decisions likewise,
+    relative to tau."""
+
+    def __init__(self):
+        self.decisions = 0          # (observation, sequence) pairs that evicted pages
+        self.pages_evicted = 0
+        self.inside_band = 0        # of those, boundary gap <= TIE_REL
+        self.gap_le = {1e-6: 0, 1e-7: 0, 0.0: 0}
+        self.evict_adoptions = 0
+        self.evict_adopt_max_dist = 0.0
+        self.tokens_observed = 0
+        self.refresh_in_band = 0    # tokens with |Abar - tau| <= TIE_REL tau
+        self.refresh_adoptions = 0  # of those, decided differently by the GPU
+        self.refresh_adopt_max_dist = 0.0
+
+    def evict(self, S, want, got, page_flip):
+        S = np.asarray(S, np.float64)
+        if not want:
+            return
+        self.decisions += 1
+        self.pages_evicted += len(want)
+        boundary = max(S[j] for j in want)
+        chosen = set(want)
+        kept = [S[j] for j in range(len(S)) if j not in chosen and np.isfinite(S[j])]
+        gap = (min(kept) - boundary) / (abs(boundary) + TOL_FLOOR) if kept else np.inf
+        gap = abs(gap)
+        if gap <= TIE_REL:
+            self.inside_band += 1
+        for x in self.gap_le:
+            if gap <= x:
+                self.gap_le[x] += 1
+        if got is not None and sorted(got) != sorted(want):
+            self.evict_adoptions += 1
+            for j in set(got) ^ chosen:
+                if not page_flip[j]:
+                    d = abs(S[j] - boundary) / (abs(boundary) + TOL_FLOOR)
+                    self.evict_adopt_max_dist = max(self.evict_adopt_max_dist, d)
+
+    def refresh(self, abar, tau, mism):
+        abar = np.asarray(abar, np.float64)
+        self.tokens_observed += len(abar)
+        self.refresh_in_band += int(np.count_nonzero(np.abs(abar - tau) <= TIE_REL * tau))
+        if mism.any():
+            self.refresh_adoptions += int(mism.sum())
+            d = float(np.max(np.abs(abar[mism] - tau))) / tau
+            self.refresh_adopt_max_dist = max(self.refresh_adopt_max_dist, d)
+
+    def merge(self, other: "TieStats"):
+        for k, v in vars(other).items():
+            if k == "gap_le":
+                for x, n in v.items():
+                    self.gap_le[x] += n
+            elif k.endswith("max_dist"):
+                setattr(self, k, max(getattr(self, k), v))
+            else:
+                setattr(self, k, getattr(self, k) + v)
+
+    def summary(self) -> dict:
+        d = {k: v for k, v in vars(self).items() if k != "gap_le"}
+        d.update({f"gap_le_{x:g}": n for x, n in self.gap_le.items()})
+        return d
+
+
 def to_dev(a: np.ndarray) -> torch.Tensor:
     """uint16 bf16 bits -> int16 device tensor (same bits)."""
     return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda()
@@ -76,6 +149,7 @@ class Lockstep:
         self.step_no = 0
         self.resyncs = {"evict": 0, "refresh": 0}
         self.max_err = {"O": 0.0, "ahat": 0.0, "a": 0.0, "prio": 0.0, "page": 0.0}
+        self.ties = TieStats()
 
     # ------------------------------------------------------------ feeding --
     def prefill(self):
@@ -160,6 +234,8 @@ class Lockstep:
             # refresh decisions: exact unless within the tie band of tau
             tau = w.tau_scale / n_pre
             mism = tref[sl] != o.t_ref[sl]
+            if observed:
+                self.ties.refresh(o.abar[sl], tau, mism)
             flipped = np.zeros(n_pre, bool)
             if mism.any():
                 amb = np.abs(o.abar[sl] - tau) <= TIE_REL * tau
@@ -187,6 +263,7 @@ class Lockstep:
             # the evicted physical ids the call reports: the pages it evicted,
             # in logical order, then -1
             assert list(evd[b, n_o[b]:]) == [-1] * (self.P_max - n_o[b]), f"evicted ids padding (seq {b})"
+            self.ties.evict(S_o, want, got, page_flip)
             if got != want:
                 self._check_valid_choice(b, S_o, page_flip, got, want)
                 assert list(evd[b, :n_o[b]]) == [pre_block[b][j] for j in got], f"evicted ids (seq {b})"

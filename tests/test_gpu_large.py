@@ -1,19 +1,28 @@
 """Full-size parity at configs 3 and 4, in the benchmark's launch
 configuration (the whole batch, 77 GB of K/V per step, on the GPU), checked
 on sampled sequences {0, B/2, B-1} that the oracle recomputes one by one: at
-the full-trace observation and at the steady observations after it.  Config 4
-is also run through the layer-by-layer entry point, with region-aligned
-pages (pages then hold different numbers of tokens) and with structured keys
-(refreshes fire).
+the full-trace observation and at the 8 steady observations after it (for
+config 3 an observation closes a window of 16 decode steps, and every decode
+step's output is compared).  Config 4 runs at every swept attention weight
+w in {0, 0.5, 1, 4}, through the layer-by-layer entry point, with
+region-aligned pages (pages then hold different numbers of tokens) and with
+structured keys (refreshes fire).
 
 Sequences are independent in every stage except the shared page pool, so the
 oracle runs a sampled sequence alone (its physical page ids differ) and the
 comparison is by logical token / logical page: attention output, Abar, a,
 clocks, token and page priorities, the evicted logical pages and the order of
-the compacted block-table row.  Tolerances as in tests/gpu_harness.py.  A
-sequence whose eviction takes another valid choice inside the tie band is
-checked up to that point (the oracle cannot adopt the GPU's choice)."""
+the compacted block-table row.  Tolerances as in tests/gpu_harness.py.
+
+The run is a lockstep: after every observation, where the GPU took another
+valid choice inside the tie band (an eviction or a refresh), the oracle's
+choice is written back into the GPU's rows of that sequence (block-table
+row, the freed ids on the free stack, page fills, token count, clocks), so
+every observation of every sampled sequence is compared; the test asserts
+that count and reports how many choices were adopted and how close to the
+boundary they were."""
 import gc
+import json
 
 import numpy as np
 import pytest
@@ -27,7 +36,7 @@ import oracle.memdecay_oracle as om  # noqa: E402
 import paper_2607_10582_gb300 as md  # noqa: E402
 import synth  # noqa: E402
 from paper_2607_10582_gb300 import build as mdbuild  # noqa: E402
-from tests.gpu_harness import TIE_REL, TOL_FLOOR, TOL_O_ABS, TOL_REL, rel_err  # noqa: E402
+from tests.gpu_harness import TIE_REL, TOL_FLOOR, TOL_O_ABS, TOL_REL, TieStats, rel_err  # noqa: E402
 
 mdbuild.build()
 synth.build()
@@ -44,91 +53,144 @@ def sizes(w, aligned):
     return P_max, P_phys
 
 
-def gpu_run(w, n_obs, samples, mode="fused"):
-    """Prefill the whole batch with the CUDA generator, then n_obs observation
-    windows of window_k decode steps each; keep, for the sampled sequences,
-    what each observation needs for the comparison."""
-    dev = torch.device("cuda")
-    B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
-    P_max, P_phys = sizes(w, mode == "aligned")
-    cache = md.Cache(L, Hq, Hkv, ps, B, P_max, P_phys,
-                     rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
-                     score_mode=w.score_mode, page_reduce=w.page_reduce,
-                     region_aligned_pages=int(mode == "aligned"))
-    for r in range(7):
-        cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
-    lib = synth.lib()
-    sflag = int(w.structured)
-    kap = (synth.ctypes.c_float * 9)(*synth.KAPPA_STRUCT) if w.structured else None
-    nmax = max(w.n0(b) for b in range(B))
-    kb = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
-    vb = torch.empty_like(kb)
-    for b in range(B):
-        rd = torch.from_numpy(w.regions[b]).to(dev)
-        assert lib.synth_fill_kv_dev(w.seed, sflag, kap, b, L, Hkv, D, 0, w.n0(b), rd.data_ptr(),
-                                     kb.data_ptr(), vb.data_ptr(), None) == 0
-        cache.append_tokens(b, w.regions[b], kb.data_ptr(), vb.data_ptr(), w.insert_steps[b])
-        torch.cuda.synchronize()
-    del kb, vb
-    q = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
-    kn = torch.empty((B, L, Hkv, D), dtype=torch.int16, device=dev)
-    vn = torch.empty_like(kn)
-    out = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
-    regs = [w.decode_region] * B
-    rdev = torch.tensor(regs, dtype=torch.uint8, device=dev)
-    obs = []
-    t = 0
-    for o in range(n_obs):
-        for k in range(w.window_k):
-            t += 1
-            pos = torch.tensor([w.n0(b) + t - 1 for b in range(B)], dtype=torch.int32, device=dev)
-            assert lib.synth_fill_q_dev(w.seed, sflag, kap, B, L, Hq, Hq // Hkv, D, t, q.data_ptr(), None) == 0
-            assert lib.synth_fill_step_kv_dev(w.seed, sflag, kap, B, L, Hkv, D, pos.data_ptr(), rdev.data_ptr(),
-                                              kn.data_ptr(), vn.data_ptr(), None) == 0
-            if mode == "layerwise":
+class GpuBatch:
+    """The whole batch on the GPU: prefill with the CUDA generator, then
+    observation windows of window_k decode steps each, keeping for the
+    sampled sequences what the comparison needs."""
+
+    def __init__(self, w, samples, mode):
+        self.w, self.samples, self.mode = w, list(samples), mode
+        dev = self.dev = torch.device("cuda")
+        B, L, Hq, Hkv, ps, D = w.B, w.L, w.Hq, w.Hkv, w.page_size, w.D
+        P_max, P_phys = sizes(w, mode == "aligned")
+        self.cache = md.Cache(L, Hq, Hkv, ps, B, P_max, P_phys,
+                              rho=w.rho, gamma=w.gamma, tau_scale=w.tau_scale, attn_weight=w.attn_weight,
+                              score_mode=w.score_mode, page_reduce=w.page_reduce,
+                              region_aligned_pages=int(mode == "aligned"))
+        for r in range(7):
+            self.cache.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
+        self.lib = synth.lib()
+        self.sflag = int(w.structured)
+        self.kap = (synth.ctypes.c_float * 9)(*synth.KAPPA_STRUCT) if w.structured else None
+        nmax = max(w.n0(b) for b in range(B))
+        kb = torch.empty(L * Hkv * nmax * D, dtype=torch.int16, device=dev)
+        vb = torch.empty_like(kb)
+        for b in range(B):
+            rd = torch.from_numpy(w.regions[b]).to(dev)
+            assert self.lib.synth_fill_kv_dev(w.seed, self.sflag, self.kap, b, L, Hkv, D, 0, w.n0(b),
+                                              rd.data_ptr(), kb.data_ptr(), vb.data_ptr(), None) == 0
+            self.cache.append_tokens(b, w.regions[b], kb.data_ptr(), vb.data_ptr(), w.insert_steps[b])
+            torch.cuda.synchronize()
+        del kb, vb
+        self.q = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+        self.kn = torch.empty((B, L, Hkv, D), dtype=torch.int16, device=dev)
+        self.vn = torch.empty_like(self.kn)
+        self.out = torch.empty((B, L, Hq, D), dtype=torch.int16, device=dev)
+        self.regs = [w.decode_region] * B
+        self.rdev = torch.tensor(self.regs, dtype=torch.uint8, device=dev)
+        self.t = 0
+
+    def window(self):
+        """window_k decode steps; returns, per sampled sequence, the output
+        of every step (bf16 bits)."""
+        w, c = self.w, self.cache
+        B, L, Hq, Hkv, D = w.B, w.L, w.Hq, w.Hkv, w.D
+        outs = {b: [] for b in self.samples}
+        for _ in range(w.window_k):
+            self.t += 1
+            pos = torch.tensor([w.n0(b) + self.t - 1 for b in range(B)], dtype=torch.int32, device=self.dev)
+            assert self.lib.synth_fill_q_dev(w.seed, self.sflag, self.kap, B, L, Hq, Hq // Hkv, D, self.t,
+                                             self.q.data_ptr(), None) == 0
+            assert self.lib.synth_fill_step_kv_dev(w.seed, self.sflag, self.kap, B, L, Hkv, D, pos.data_ptr(),
+                                                   self.rdev.data_ptr(), self.kn.data_ptr(), self.vn.data_ptr(),
+                                                   None) == 0
+            if self.mode == "layerwise":
                 # a model hands each layer its own contiguous [B][heads][D] tensors
                 for l in range(L):
-                    ol = torch.empty((B, Hq, D), dtype=torch.int16, device=dev)
-                    cache.decode_layer(l, B, q[:, l].contiguous(), kn[:, l].contiguous(),
-                                       vn[:, l].contiguous(), regs, ol)
-                    out[:, l] = ol
+                    ol = torch.empty((B, Hq, D), dtype=torch.int16, device=self.dev)
+                    c.decode_layer(l, B, self.q[:, l].contiguous(), self.kn[:, l].contiguous(),
+                                   self.vn[:, l].contiguous(), self.regs, ol)
+                    self.out[:, l] = ol
             else:
-                cache.decode_step(B, q, kn, vn, regs, out)
-        o_last = out.cpu().numpy().view(np.uint16)
-        pre_bt = cache.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
-        pre_fill = cache.get_state(md.MD_STATE_PAGE_FILL).cpu().numpy()
-        pre_pages = [cache.query(md.MD_QUERY_PAGES, b) for b in range(B)]
-        pre_tokens = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
-        st, n_ev = cache.evict(w.budget_pages)
+                c.decode_step(B, self.q, self.kn, self.vn, self.regs, self.out)
+            o_h = self.out.cpu().numpy().view(np.uint16)
+            for b in self.samples:
+                outs[b].append(o_h[b].copy())
+        return outs
+
+    def observe(self):
+        """md_evict over the batch; returns per sampled sequence the state the
+        comparison reads, by logical token / page."""
+        w, c = self.w, self.cache
+        B, ps = w.B, w.page_size
+        pre_bt = c.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
+        pre_fill = c.get_state(md.MD_STATE_PAGE_FILL).cpu().numpy()
+        pre_pages = [c.query(md.MD_QUERY_PAGES, b) for b in range(B)]
+        pre_tokens = [c.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+        st, n_ev = c.evict(w.budget_pages)
         torch.cuda.synchronize()
-        assert cache.sync() == md.MD_OK
-        st_arr = {name: cache.get_state(what).cpu().numpy()
+        assert c.sync() == md.MD_OK
+        self.n_ev = [int(x) for x in n_ev]
+        st_arr = {name: c.get_state(what).cpu().numpy()
                   for name, what in (("ahat", md.MD_STATE_AHAT), ("a", md.MD_STATE_A),
                                      ("t_ref", md.MD_STATE_T_REF), ("prio", md.MD_STATE_TOKEN_PRIO),
                                      ("page", md.MD_STATE_PAGE_SCORE), ("bt", md.MD_STATE_BLOCK_TABLE))}
         rec = {}
-        for b in samples:
-            n_pre = pre_tokens[b]
-            P = pre_pages[b]
-            fills = [int(pre_fill[b, j]) if mode == "aligned" else min(ps, n_pre - j * ps) for j in range(P)]
+        for b in self.samples:
+            n_pre, P = pre_tokens[b], pre_pages[b]
+            fills = [int(pre_fill[b, j]) for j in range(P)]
+            assert sum(fills) == n_pre
             gsl = np.array([pre_bt[b, j] * ps + o for j in range(P) for o in range(fills[j])])
-            assert len(gsl) == n_pre
-            rec[b] = dict(n_ev=int(n_ev[b]), n_pre=n_pre, out=o_last[b].copy(), pre_bt=pre_bt[b, :P].copy(),
-                          ahat=st_arr["ahat"][gsl], a=st_arr["a"][gsl], t_ref=st_arr["t_ref"][gsl],
-                          prio=st_arr["prio"][gsl], page=st_arr["page"][b, :P].copy(),
-                          bt=st_arr["bt"][b, :P].copy())
-        obs.append(rec)
-        del st_arr
-    cache.close()
-    del cache, q, kn, vn, out
-    gc.collect()
-    torch.cuda.empty_cache()
-    return obs
+            rec[b] = dict(n_ev=self.n_ev[b], n_pre=n_pre, gsl=gsl, pre_bt=pre_bt[b, :P].copy(),
+                          pre_fill=np.array(fills), ahat=st_arr["ahat"][gsl], a=st_arr["a"][gsl],
+                          t_ref=st_arr["t_ref"][gsl], prio=st_arr["prio"][gsl],
+                          page=st_arr["page"][b, :P].copy(), bt=st_arr["bt"][b, :P].copy())
+        return rec
+
+    def adopt_eviction(self, b, g, want):
+        """Write the oracle's eviction (logical pages `want`) into sequence b's
+        rows: the compacted block-table row and fills, the freed ids in the
+        free-stack segment where this observation pushed b's pages (pushes go
+        in sequence order from the pre-eviction top), the token count."""
+        c = self.cache
+        bt = c.get_state(md.MD_STATE_BLOCK_TABLE).cpu().numpy()
+        fill = c.get_state(md.MD_STATE_PAGE_FILL).cpu().numpy()
+        free = c.get_state(md.MD_STATE_FREE).cpu().numpy()
+        ntok = c.get_state(md.MD_STATE_SEQ_TOKENS).cpu().numpy()
+        P = len(g["pre_bt"])
+        gone = set(want)
+        kept = [j for j in range(P) if j not in gone]
+        bt[b, :] = -1
+        bt[b, :len(kept)] = g["pre_bt"][kept]
+        fill[b, :] = 0
+        fill[b, :len(kept)] = g["pre_fill"][kept]
+        top = c.query(md.MD_QUERY_FREE_TOP)
+        seg = top - sum(self.n_ev) + sum(self.n_ev[:b])
+        free[seg:seg + len(want)] = g["pre_bt"][sorted(want)]
+        ntok[b] = g["n_pre"] - int(g["pre_fill"][sorted(want)].sum())
+        for what, arr in ((md.MD_STATE_BLOCK_TABLE, bt), (md.MD_STATE_PAGE_FILL, fill),
+                          (md.MD_STATE_FREE, free), (md.MD_STATE_SEQ_TOKENS, ntok)):
+            c.set_state(what, torch.from_numpy(arr).cuda())
+        torch.cuda.synchronize()
+
+    def adopt_refresh(self, g, mism, t_ref_oracle):
+        c = self.cache
+        t_ref = c.get_state(md.MD_STATE_T_REF).cpu().numpy()
+        t_ref[g["gsl"][mism]] = t_ref_oracle[mism]
+        c.set_state(md.MD_STATE_T_REF, torch.from_numpy(t_ref.astype(np.int32)).cuda())
+        torch.cuda.synchronize()
+
+    def close(self):
+        self.cache.close()
+        del self.cache, self.q, self.kn, self.vn, self.out
+        gc.collect()
+        torch.cuda.empty_cache()
 
 
 def oracle_run(w, b, n_obs, aligned=False):
-    """The oracle for sequence b alone, same inputs, same schedule; yields one
-    record per observation."""
+    """The oracle for sequence b alone, same inputs, same schedule; yields,
+    per observation, the outputs of the window's decode steps and the state
+    after the observation."""
     n = w.n0(b)
     P_max, _ = sizes(w, aligned)
     spans = int(np.count_nonzero(np.diff(w.regions[b].astype(np.int16)))) + 2 if aligned else 0
@@ -144,34 +206,35 @@ def oracle_run(w, b, n_obs, aligned=False):
     del k, v
     t = 0
     for _ in range(n_obs):
+        Os = []
         for _k in range(w.window_k):
             t += 1
             q = synth.q_host(w.seed, w.B, w.L, w.Hq, w.Hkv, t, w.structured)[b:b + 1]
             kn, vn = synth.kv_host(w.seed, b, w.L, w.Hkv, n + t - 1, 1, np.array([w.decode_region], np.uint8),
                                    w.structured)
-            O = o.decode_step(1, q, kn[:, :, 0, :][None], vn[:, :, 0, :][None], [w.decode_region])
-        pre_block = list(o.block[0])
-        pre_slots = o.slots(0)
+            Os.append(o.decode_step(1, q, kn[:, :, 0, :][None], vn[:, :, 0, :][None], [w.decode_region])[0])
+        osl = o.slots(0)
         pre_pot = o.page_of_token(0)
         st, n_ev, ids, logical = o.evict(1, [w.budget_pages[b]])
-        yield o, O[0], pre_block, pre_slots, pre_pot, n_ev[0], logical[0]
+        yield o, Os, osl, pre_pot, n_ev[0], logical[0]
 
 
-def compare(w, g, o, O, pre_block, osl, pre_pot, ne_o, logical_o, where):
-    """One observation of one sampled sequence; returns False when the GPU
-    took another valid choice inside the tie band (the trajectories part)."""
-    ps = w.page_size
+def compare(w, g, outs, o, Os, osl, pre_pot, ne_o, logical_o, where, ties):
+    """One observation of one sampled sequence.  Returns (the evicted logical
+    pages the GPU chose, the tokens whose refresh decision differs)."""
     assert g["n_ev"] == ne_o, where
-    err = float(np.max(np.abs(synth.bf16_to_f64(g["out"]) - O)))
-    assert err <= TOL_O_ABS, (where, err)
+    for k, (gout, O) in enumerate(zip(outs, Os)):
+        err = float(np.max(np.abs(synth.bf16_to_f64(gout) - O)))
+        assert err <= TOL_O_ABS, (where, k, err)
     assert g["n_pre"] == len(osl), where
-    P = len(pre_block)
+    P = len(g["pre_bt"])
     for key, arr in (("ahat", o.abar), ("a", o.a)):
         e = rel_err(g[key], arr[osl])
         assert e <= TOL_REL, (where, key, e)
     tau = w.tau_scale / g["n_pre"]
     mism = g["t_ref"] != o.t_ref[osl]
     assert np.all(np.abs(o.abar[osl][mism] - tau) <= TIE_REL * tau), (where, "refresh")
+    ties.refresh(o.abar[osl], tau, mism)
     e = rel_err(g["prio"][~mism], o.prio[osl][~mism])
     assert e <= TOL_REL, (where, "prio", e)
     page_flip = np.zeros(P, bool)
@@ -182,30 +245,52 @@ def compare(w, g, o, O, pre_block, osl, pre_pot, ne_o, logical_o, where):
     kept = g["bt"][:P - ne_o]
     got = sorted(int(j) for j in np.nonzero(~np.isin(g["pre_bt"], kept))[0])
     assert list(kept) == [g["pre_bt"][j] for j in range(P) if j not in set(got)], where
+    ties.evict(S_o, logical_o, got, page_flip)
     if got != logical_o:
         boundary = max(S_o[j] for j in logical_o)
         for j in set(got) ^ set(logical_o):
             assert page_flip[j] or abs(S_o[j] - boundary) <= TIE_REL * abs(boundary) + TOL_FLOOR, where
-        return False
-    return not mism.any()
+    return got, mism
 
 
-@pytest.mark.parametrize("config,w_attn,n_obs,mode", [(4, 1.0, 9, "fused"), (3, 1.0, 2, "fused"),
-                                                     (4, 0.0, 3, "fused"), (4, 4.0, 3, "fused"),
-                                                     (4, 1.0, 3, "layerwise"), (4, 1.0, 3, "aligned"),
-                                                     (4, 1.0, 3, "structured")])
-def test_full_size_sampled_sequences(config, w_attn, n_obs, mode):
+CASES = [(4, 1.0, "fused"), (3, 1.0, "fused"), (4, 0.0, "fused"), (4, 0.5, "fused"), (4, 4.0, "fused"),
+         (4, 1.0, "layerwise"), (4, 1.0, "aligned"), (4, 1.0, "structured")]
+N_OBS = 9   # the full-trace observation and 8 steady ones
+
+
+@pytest.mark.parametrize("config,w_attn,mode", CASES)
+def test_full_size_sampled_sequences(config, w_attn, mode):
     w = synth.make_workload(config, attn_weight=w_attn, structured=(mode == "structured"))
-    samples = (0, w.B // 2, w.B - 1) if (w_attn == 1.0 and mode == "fused") else (w.B // 2,)
-    obs = gpu_run(w, n_obs, samples, mode)
+    samples = (0, w.B // 2, w.B - 1)
+    gpu = GpuBatch(w, samples, mode)
+    runs = {b: oracle_run(w, b, N_OBS, aligned=(mode == "aligned")) for b in samples}
+    ties = TieStats()
+    compared = {b: 0 for b in samples}
+    adopted = {b: {"evict": 0, "refresh": 0} for b in samples}
     refreshed = 0
-    for b in samples:
-        runs = oracle_run(w, b, n_obs, aligned=(mode == "aligned"))
-        for i, (o, O, pre_block, osl, pre_pot, ne_o, logical_o) in enumerate(runs):
+    for i in range(N_OBS):
+        outs = gpu.window()
+        rec = gpu.observe()
+        for b in samples:
+            o, Os, osl, pre_pot, ne_o, logical_o = next(runs[b])
             refreshed += int(np.count_nonzero((o.t_ref[osl] == o.t) & (o.t_ins[osl] < o.t)))
-            if not compare(w, obs[i][b], o, O, pre_block, osl, pre_pot, ne_o, logical_o,
-                           (config, w_attn, mode, b, i)):
-                break           # another valid choice inside the tie band: trajectories part here
+            got, mism = compare(w, rec[b], outs[b], o, Os, osl, pre_pot, ne_o, logical_o,
+                                (config, w_attn, mode, b, i), ties)
+            compared[b] += 1
+            if got != logical_o:
+                gpu.adopt_eviction(b, rec[b], logical_o)
+                adopted[b]["evict"] += 1
+            if mism.any():
+                gpu.adopt_refresh(rec[b], mism, o.t_ref[osl])
+                adopted[b]["refresh"] += int(mism.sum())
         gc.collect()
+    gpu.close()
+    for b in samples:
+        runs[b].close()
+    report = {"config": config, "w": w_attn, "mode": mode, "observations_compared": compared,
+              "adopted": adopted, "ties": ties.summary(), "refreshed_tokens": refreshed}
+    print("\nFULL-SIZE PARITY " + json.dumps(report))
+    assert all(n == N_OBS for n in compared.values()), compared
+    assert ties.decisions >= len(samples)          # the full-trace observation evicts in every sequence
     if mode == "structured":
         assert refreshed > 0   # the structured keys make Eq. 3's refresh fire

@@ -1,5 +1,7 @@
 """GPU parity: the CUDA path, called through the C ABI, against the fp64
 oracle on the same seeded inputs (tolerances in tests/gpu_harness.py)."""
+import json
+
 import numpy as np
 import pytest
 
@@ -40,12 +42,20 @@ def test_cuda_generator_matches_host():
     assert np.array_equal(qd.cpu().numpy().view(np.uint16), q)
 
 
+def report(name, ls):
+    """One line per lockstep run: largest errors, the choices adopted inside
+    the tie band and how close the decisions came to the band (TieStats)."""
+    print("\nLOCKSTEP " + json.dumps({"run": name, "max_err": ls.max_err, "resyncs": ls.resyncs,
+                                      "ties": ls.ties.summary()}))
+
+
 def test_config0_full_run():
     """Config 0 end to end: 448-token trace, 64 decode steps, eviction to 50%
     of pages at every step."""
     ls = Lockstep(synth.make_workload(0)).run()
     ls.check_layout()
     assert ls.max_err["O"] < 2e-2
+    report("config 0", ls)
 
 
 def test_multichunk_ragged_batch():
@@ -198,27 +208,25 @@ def test_config1_full_run():
     ls = Lockstep(synth.make_workload(1))
     ls.run()
     ls.check_layout()
+    report("config 1", ls)
 
 
-def test_config2_first_steps():
-    """Config 2 geometry (Qwen2.5-3B, 36 layers, 16/2), 32 sequences with
-    Dirichlet region spans and insertion offsets: the full-trace step and 31
-    steady steps, every sequence at every step (two page boundaries pass, so
-    appends take pages the evictions freed)."""
-    ls = Lockstep(synth.make_workload(2))
-    ls.run(steps=32)
+@pytest.mark.parametrize("structured", [False, True])
+def test_config2_all_steps(structured):
+    """Config 2 end to end (Qwen2.5-3B geometry, 36 layers, 16/2 heads), 32
+    sequences with Dirichlet region spans and insertion offsets: the
+    full-trace step and all 255 steady steps, every sequence at every step
+    (page boundaries pass, so appends take pages the evictions freed).  With
+    structured keys and queries (per-region offsets, hot tokens) refreshes
+    fire."""
+    ls = Lockstep(synth.make_workload(2, structured=structured))
+    ls.run()
     ls.check_layout()
-
-
-def test_config2_structured():
-    """Config 2 with structured keys and queries (per-region offsets, hot
-    tokens): refreshes fire, every sequence checked at every step."""
-    ls = Lockstep(synth.make_workload(2, structured=True))
-    ls.run(steps=12)
-    ls.check_layout()
-    o = ls.orc
-    sl = np.concatenate([o.slots(b) for b in range(ls.w.B)])
-    assert np.count_nonzero((o.t_ref[sl] == o.t) & (o.t_ins[sl] < o.t)) > 0   # refreshed, not new
+    report(f"config 2{' structured' if structured else ''}", ls)
+    if structured:
+        o = ls.orc
+        sl = np.concatenate([o.slots(b) for b in range(ls.w.B)])
+        assert np.count_nonzero((o.t_ref[sl] == o.t) & (o.t_ins[sl] < o.t)) > 0   # refreshed, not new
 
 
 def _small_run(seed):

@@ -396,9 +396,15 @@ def oracle_sample(w, layers: int, seq: int = 0):
         o.set_region_params(r, w.base[r], w.half_life[r], bool(w.pinned[r]))
     k, v = synth.kv_host(w.seed, seq, layers, w.Hkv, 0, n, w.regions[seq], w.structured)
     o.append_tokens(0, w.regions[seq], k, v, w.insert_steps[seq])
-    q = synth.q_host(w.seed, 1, layers, w.Hq, w.Hkv, 1, w.structured)
-    kn, vn = synth.step_kv_host(w.seed, [n], [w.decode_region], layers, w.Hkv, w.structured)
-    return o, (q, kn, vn)
+    return o
+
+
+def oracle_step_inputs(w, layers: int, seq: int, t: int):
+    """Queries and the new token's K/V of decode step t for one sequence."""
+    import synth
+    q = synth.q_host(w.seed, w.B, layers, w.Hq, w.Hkv, t, w.structured)[seq:seq + 1]
+    kn, vn = synth.step_kv_host(w.seed, [w.n0(seq) + t - 1], [w.decode_region], layers, w.Hkv, w.structured)
+    return q, kn, vn
 
 
 def make_workload(args, seed):
@@ -416,39 +422,69 @@ def make_workload(args, seed):
 
 
 def _oracle_worker(task):
-    """One host process: the oracle on one sampled sequence (layers of L
-    layers), prefilled once, then `reps` timed steps (each on a fresh copy of
-    the prefilled state).  Returns per-step (decode seconds, evict seconds)."""
+    """One host process: the oracle on one sampled sequence (`layers` of its
+    L layers).  Full-trace phase: prefilled once, then `reps` timed steps,
+    each on a fresh copy of the prefilled state.  Steady phase: the first
+    observation window (the full-trace step and the eviction to budget) runs
+    untimed, then `reps` windows of window_k decode steps and their
+    observation are timed.  Returns per step (decode seconds, evict seconds):
+    a window's times divided by its decode steps."""
     args_d, seq, layers, reps = task
     a = argparse.Namespace(**args_d)
     w = make_workload(a, a.seed)
-    o0, inputs = oracle_sample(w, layers, seq)
+    o0 = oracle_sample(w, layers, seq)
     out = []
+    if a.phase == "steady":
+        o, t = o0, 0
+
+        def window():
+            nonlocal t
+            dec, tok = 0.0, 0
+            for _ in range(w.window_k):
+                t += 1
+                q, kn, vn = oracle_step_inputs(w, layers, seq, t)
+                t0 = time.perf_counter()
+                o.decode_step(1, q, kn, vn, [w.decode_region])
+                dec += time.perf_counter() - t0
+                tok += o.n_tokens[0]
+            t0 = time.perf_counter()
+            o.evict(1, [w.budget_pages[seq]])
+            return dec, time.perf_counter() - t0, tok
+
+        window()
+        for _ in range(reps):
+            dec, ev, tok = window()
+            out.append((dec / w.window_k, ev / w.window_k, tok / w.window_k))
+        return out
+    q, kn, vn = oracle_step_inputs(w, layers, seq, 1)
     for _ in range(reps):
         o = copy.deepcopy(o0)
-        q, kn, vn = inputs
         t0 = time.perf_counter()
         o.decode_step(1, q, kn, vn, [w.decode_region])
         t1 = time.perf_counter()
         o.evict(1, [w.budget_pages[seq]])
         t2 = time.perf_counter()
-        out.append((t1 - t0, t2 - t1))
+        out.append((t1 - t0, t2 - t1, w.n0(seq) + 1))
     return out
 
 
-ORACLE_SAMPLE_LAYERS = 8   # layers of the oracle's bounded sample (a few seconds per process)
+ORACLE_SAMPLE_LAYERS = 8       # layers of the oracle's sample on a long full trace
+ORACLE_ALL_LAYERS_TOKENS = 8192   # traces up to this long run every layer
 
 
-def parallel_oracle(args, reps: int, layers: int = ORACLE_SAMPLE_LAYERS):
+def parallel_oracle(args, reps: int):
     """Time the fp64 oracle on the host cores: one process per core (numpy
     single-threaded in each), each on its own sequence of the workload.  The
     whole workload's step time is ceil(B / P) times the slowest process's
-    step, with the decode part scaled from `layers` to all L layers (the
-    attention work is linear in L).  Returns (seconds per step for each rep,
-    processes, sample text)."""
+    step.  On the full-trace step of a long trace the oracle attends over
+    ORACLE_SAMPLE_LAYERS layers and its decode time is scaled to all L layers
+    (the attention work is linear in L); otherwise every layer runs.  Returns
+    (seconds per step for each rep as measured on the sample, seconds per step
+    scaled to the workload for each rep, processes, a description)."""
     import multiprocessing as mp
     w = make_workload(args, args.seed)
-    layers = max(1, min(layers, w.L))
+    long_full = args.phase == "full" and w.n0(0) > ORACLE_ALL_LAYERS_TOKENS
+    layers = min(ORACLE_SAMPLE_LAYERS, w.L) if long_full else w.L
     try:
         ncpu = len(os.sched_getaffinity(0))
     except AttributeError:
@@ -462,28 +498,45 @@ def parallel_oracle(args, reps: int, layers: int = ORACLE_SAMPLE_LAYERS):
     with ctx.Pool(P) as pool:
         res = pool.map(_oracle_worker, tasks)
     rounds = -(-w.B // P)
-    per_rep = []
+    measured, scaled = [], []
     for r in range(reps):
-        slowest = max(d * (w.L / layers) + e for (d, e) in (res[p][r] for p in range(P)))
-        per_rep.append(rounds * slowest)
-    sample = (f"sequences 0..{P - 1} of {w.B}, one per process on {P} host cores (single-threaded "
-              f"numpy), {layers} of {w.L} layers of the full trace ({w.n0(0)} tokens each): decode time "
-              f"x{w.L / layers:g} + observation/eviction, x{rounds} rounds")
-    return per_rep, P, sample
+        measured.append(max(d + e for (d, e, _) in (res[p][r] for p in range(P))))
+        scaled.append(rounds * max(d * (w.L / layers) + e for (d, e, _) in (res[p][r] for p in range(P))))
+    # cached tokens per step of the whole batch: the measured sequences' mean
+    # per sequence (exact in the full-trace phase, where every sequence of a
+    # config holds the same trace length)
+    tokens_step = w.B * float(np.mean([x[2] for p in range(P) for x in res[p]]))
+    what = ("the full-trace step (prefill untimed, the state copied before each step)" if args.phase == "full"
+            else f"steady steps: the first observation window (full trace, eviction to budget) untimed, then "
+                 f"windows of {w.window_k} decode step(s) and their observation, per decode step")
+    scale = []
+    if layers < w.L:
+        scale.append(f"decode time x{w.L / layers:g} ({layers} of {w.L} layers measured)")
+    if rounds > 1:
+        scale.append(f"x{rounds} rounds ({P} of {w.B} sequences measured)")
+    sample = (f"sequences 0..{P - 1} of {w.B}, one per process on {P} host cores (single-threaded numpy), "
+              f"{w.n0(0)}-token traces, {what}; " +
+              ("measured on the whole workload" if not scale else "scaled to the workload: " + "; ".join(scale)))
+    info = {"processes": P, "layers_measured": layers, "layers": w.L, "rounds": rounds, "sample": sample,
+            "scaled": bool(scale), "tokens_per_step": tokens_step}
+    return measured, scaled, info
 
 
 def run_reference(args):
     w = make_workload(args, args.seed)
-    tokens_step = sum(w.n0(b) + 1 for b in range(w.B))
-    per_rep, cores, sample = parallel_oracle(args, args.warmup + args.steps)
-    sec = float(np.mean(per_rep[args.warmup:]))
-    value = tokens_step / sec
+    measured, scaled, info = parallel_oracle(args, args.warmup + args.steps)
+    sec = float(np.mean(scaled[args.warmup:]))
+    value = info["tokens_per_step"] / sec
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+            "ms_per_step_kind": ("scaled to the workload from a measured sample (see cpu_baseline.sample)"
+                                 if info["scaled"] else "measured"),
+            "measured_sample_ms_per_step": float(np.mean(measured[args.warmup:])) * 1e3,
+            "scaled_from_layers": info["layers_measured"] if info["layers_measured"] < info["layers"] else None,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(w, args),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": info["processes"], "kind": "oracle",
+                             "sample": info["sample"]},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -593,9 +646,16 @@ def main():
                        "entry": ("pinned-host copies + md_decode_layer x L + md_evict" if args.layerwise
                                  else "md_decode_step_host (host buffers, copies in the call) + md_evict")}
     if not args.no_cpu_baseline and world == 1:
-        per_rep, cores, sample = parallel_oracle(args, 3)
-        line["cpu_baseline"] = {"value": sum(w.n0(b) + 1 for b in range(w.B)) / min(per_rep), "unit": UNIT,
-                                "cores": cores, "kind": "oracle", "sample": sample}
+        measured, scaled, info = parallel_oracle(args, 3)
+        line["cpu_baseline"] = {"value": info["tokens_per_step"] / min(scaled), "unit": UNIT,
+                                "cores": info["processes"],
+                                "kind": "oracle", "sample": info["sample"],
+                                "ms_per_step": min(scaled) * 1e3,
+                                "ms_per_step_kind": "scaled from the measured sample" if info["scaled"]
+                                else "measured",
+                                "measured_sample_ms_per_step": min(measured) * 1e3,
+                                "scaled_from_layers": info["layers_measured"]
+                                if info["layers_measured"] < info["layers"] else None}
     print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

@@ -29,3 +29,23 @@ def test_clock_summary_falls_back_and_says_so():
 
 def test_clock_summary_without_samples_is_none():
     assert bench.ClockSampler(0).summarise(0.0, 1.0) is None
+
+
+def _args(phase):
+    return dict(config=0, w=1.0, phase=phase, seed=0, max_tokens=0, structured=False)
+
+
+def test_oracle_baseline_times_the_phase_it_names():
+    """The CPU baseline's steady phase times steps at budget occupancy (the
+    first window, full trace and eviction, runs untimed); the full-trace
+    phase times the first step over the whole trace."""
+    import synth
+    w = synth.make_workload(0)
+    full = bench._oracle_worker((_args("full"), 0, w.L, 2))
+    assert len(full) == 2 and all(tok == w.n0(0) + 1 for _, _, tok in full)
+    steady = bench._oracle_worker((_args("steady"), 0, w.L, 2))
+    assert len(steady) == 2
+    cap = w.budget_pages[0] * w.page_size
+    for dec, ev, tok in steady:
+        assert dec > 0 and ev > 0
+        assert cap - w.page_size < tok <= cap + 1    # at the budget, not the whole trace

@@ -300,13 +300,17 @@ md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_p
  *                             attention work planner adds to each chunk
  *                             (default 112; 0..65536)
  *   MD_DEBUG_FORCE_CHUNKS     chunks per (sequence, layer, KV head) item
- *                             (0 = planned; otherwise clamped to the limits) */
+ *                             (0 = planned; otherwise clamped to the limits)
+ *   MD_DEBUG_COMBINE_OVERHEAD cost, in KiB of K/V streamed by one CTA, that
+ *                             the planner adds to a split giving any item
+ *                             several chunks (default 192; 0..65536) */
 enum {
   MD_DEBUG_SPIN_LIMIT_NS = 0,
   MD_DEBUG_EXTRA_ARRIVALS = 1,
   MD_DEBUG_GRID_LIMIT = 2,
   MD_DEBUG_UNIT_OVERHEAD = 3,
-  MD_DEBUG_FORCE_CHUNKS = 4
+  MD_DEBUG_FORCE_CHUNKS = 4,
+  MD_DEBUG_COMBINE_OVERHEAD = 5
 };
 md_status md_debug_set(md_ctx *ctx, int key, int64_t value);
 

@@ -67,9 +67,13 @@ struct Unit {
 
 __device__ __forceinline__ Unit decode_unit(const AttnParams &p, int u) {
   int lo = 0, hi = p.n_seqs - 1;
-  while (lo < hi) {
-    int mid = (lo + hi + 1) >> 1;
-    if (p.unit_start[mid] <= u) lo = mid; else hi = mid - 1;
+  if (p.units_per_seq > 0) {          // every sequence has the same number of units
+    lo = u / p.units_per_seq;
+  } else {
+    while (lo < hi) {
+      int mid = (lo + hi + 1) >> 1;
+      if (p.unit_start[mid] <= u) lo = mid; else hi = mid - 1;
+    }
   }
   Unit un;
   un.b = lo;
@@ -85,6 +89,27 @@ __device__ __forceinline__ Unit decode_unit(const AttnParams &p, int u) {
   un.p1 = (int)(((long long)(un.j + 1) * P) / un.C);
   un.X = (lo * p.L + un.l) * p.Hkv + un.kvh;
   return un;
+}
+
+/* Physical ids (and, with region-aligned pages, fills) of pages [from,
+ * from + 8) of unit x, cut at the unit's end; returns how many.  The loads
+ * are independent, so all of them are in flight at once. */
+template <bool ALIGNED>
+__device__ __forceinline__ int load_batch(const AttnParams &p, const Unit &x, int from, int (&ph)[8],
+                                          int (&fl)[8]) {
+  const int cnt = min(8, x.p1 - from);
+  const int32_t *bt = p.block_table + (size_t)x.b * p.P_max;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) ph[k] = k < cnt ? bt[from + k] : 0;
+  if (ALIGNED) {
+    const uint8_t *fr = p.page_fill + (size_t)x.b * p.P_max;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) fl[k] = k < cnt ? fr[from + k] : 0;
+  } else {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) fl[k] = 0;
+  }
+  return cnt;
 }
 
 __device__ __forceinline__ void raise_status(const AttnParams &p, int code, int diag) {
@@ -481,6 +506,10 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     fence_barrier_init();
   }
   __syncthreads();
+  /* the kernel ahead in the stream (append) writes the pool, the block table
+   * and the page fills this one reads */
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     /* ------------------------------------------------------- producer ---- */
@@ -494,57 +523,79 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
        * i % NCW: R is a multiple of NCW, so every stage belongs to one warp */
       int i = 0, nu = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-        const Unit un = decode_unit(p, u);
-        /* the unit's G query rows: one bulk copy into a double-buffered slot */
-        const int qs = nu & 1;
-        if (nu >= 2) {
-          if (!wait_phase(smem_u32(&qempty[qs]), ((nu >> 1) - 1) & 1, p, 5, true)) {
-            ok = false;
-            break;
+      /* The CTA's pages as one stream of batches of up to 8 pages (never
+       * across a unit); the page ids (and fills) of the next batch are loaded
+       * before the current batch's copies are issued, so their latency hides
+       * behind the waits for free stages instead of emptying the ring. */
+      int u = blockIdx.x;
+      Unit un{};
+      int pb = 0, cnt = 0;
+      int ph[8], fl[8];
+      if (u < p.total_units) {
+        un = decode_unit(p, u);
+        pb = un.p0;
+        cnt = load_batch<ALIGNED>(p, un, pb, ph, fl);
+      }
+      while (u < p.total_units && ok) {
+        Unit nx = un;
+        int npb = pb + 8, nxu = u, cntn = 0;
+        int phn[8] = {0, 0, 0, 0, 0, 0, 0, 0}, fln[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        if (npb >= un.p1) {
+          nxu = u + gridDim.x;
+          if (nxu < p.total_units) {
+            nx = decode_unit(p, nxu);
+            npb = nx.p0;
           }
-          /* the consumers read the slot through the generic proxy; the bulk
-           * copy writes it through the async proxy */
-          fence_proxy_async_smem();
         }
-        mbar_arrive_expect_tx(smem_u32(&qfull[qs]), G * D * 2);
-        bulk_load(sQ_u32 + qs * S::Q_BYTES,
-                  p.q + (((size_t)un.b * p.q_layers + (un.l - p.l0)) * p.Hq + (size_t)un.kvh * G) * D, G * D * 2,
-                  smem_u32(&qfull[qs]));
-        ++nu;
-        const int32_t *bt = p.block_table + (size_t)un.b * p.P_max;
-        for (int pb = un.p0; pb < un.p1 && ok; pb += 8) {
-          const int cnt = min(8, un.p1 - pb);
-          int ph[8], fl[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) ph[k] = k < cnt ? bt[pb + k] : 0;
-          if (ALIGNED) {
-            const uint8_t *fr = p.page_fill + (size_t)un.b * p.P_max;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) fl[k] = k < cnt ? fr[pb + k] : 0;
-          }
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            if (k >= cnt) break;
-            const int s = i % S::R;
-            if (i >= S::R) {
-              if (!wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
-                ok = false;
-                break;
-              }
-              /* the stage's last reads (ldmatrix, generic proxy) must be
-               * ordered before the TMA refill (async proxy): without this
-               * fence a refill can overwrite V rows still being read */
-              fence_proxy_async_smem();
+        if (nxu < p.total_units) cntn = load_batch<ALIGNED>(p, nx, npb, phn, fln);
+        if (pb == un.p0) {
+          /* the unit's G query rows: one bulk copy into a double-buffered slot */
+          const int qs = nu & 1;
+          if (nu >= 2) {
+            if (!wait_phase(smem_u32(&qempty[qs]), ((nu >> 1) - 1) & 1, p, 5, true)) {
+              ok = false;
+              break;
             }
-            const int row = (((un.l * p.P_phys + ph[k]) * p.Hkv + un.kvh) * 2) * PS;
-            const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
-            if (ALIGNED) fillbuf[s] = fl[k];   // published by the arrive below
-            mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
-            tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
-            tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
-            ++i;
+            /* the consumers read the slot through the generic proxy; the bulk
+             * copy writes it through the async proxy */
+            fence_proxy_async_smem();
           }
+          mbar_arrive_expect_tx(smem_u32(&qfull[qs]), G * D * 2);
+          bulk_load(sQ_u32 + qs * S::Q_BYTES,
+                    p.q + (((size_t)un.b * p.q_layers + (un.l - p.l0)) * p.Hq + (size_t)un.kvh * G) * D,
+                    G * D * 2, smem_u32(&qfull[qs]));
+          ++nu;
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (k >= cnt) break;
+          const int s = i % S::R;
+          if (i >= S::R) {
+            if (!wait_phase(smem_u32(&empty[s]), ((i / S::R) - 1) & 1, p, 1, true)) {
+              ok = false;
+              break;
+            }
+            /* the stage's last reads (ldmatrix, generic proxy) must be
+             * ordered before the TMA refill (async proxy): without this
+             * fence a refill can overwrite V rows still being read */
+            fence_proxy_async_smem();
+          }
+          const int row = (((un.l * p.P_phys + ph[k]) * p.Hkv + un.kvh) * 2) * PS;
+          const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
+          if (ALIGNED) fillbuf[s] = fl[k];   // published by the arrive below
+          mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
+          tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
+          tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
+          ++i;
+        }
+        un = nx;
+        pb = npb;
+        u = nxu;
+        cnt = cntn;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          ph[k] = phn[k];
+          fl[k] = fln[k];
         }
       }
       /* No copy may still be writing this CTA's shared memory when it exits:
@@ -807,11 +858,13 @@ static cudaError_t launch_impl(const AttnParams &p, const CUtensorMap &tmap, int
   cfg.blockDim = dim3(AttnShape<PS, NCW>::THREADS);
   cfg.dynamicSmemBytes = AttnShape<PS, NCW>::SMEM;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, attn_mass_kernel<PS, NCW, AL>, p, tmap);
 }
 
@@ -1024,6 +1077,9 @@ extern "C" __attribute__((visibility("default"))) md_status md_attend_mass_noall
   ap.unit_start[batch] = (int)U;
   ap.total_units = (int)U;
   ap.n_seqs = batch;
+  ap.units_per_seq = (int)(U / batch);
+  for (int b = 0; b < batch && ap.units_per_seq > 0; ++b)
+    if (ap.unit_start[b + 1] - ap.unit_start[b] != ap.units_per_seq) ap.units_per_seq = 0;
 
   uint8_t *s8 = (uint8_t *)base;
   ap.status = (int *)s8;

@@ -65,12 +65,13 @@ struct md_ctx {
   int extra_arrivals = 0;
   int grid_cap = 0;          // 0: every CTA that fits
   int unit_overhead_kib = 112;   // planner: per-unit cost, as KiB of K/V streamed
+  int combine_overhead_kib = 192;   // planner: cost of a split into several chunks per item
   int force_chunks = 0;      // planner: 0 = choose
   /* the planner's last choice of pages per chunk, reused while its inputs
    * (batch, layers, knobs, pages per sequence) repeat */
   std::vector<int> plan_pages;
   int plan_batch = -1, plan_layers = -1, plan_T = 0, plan_G = 0;
-  int plan_knobs[4] = {-1, -1, -1, -1};
+  int plan_knobs[5] = {-1, -1, -1, -1, -1};
   bool calib_on = false;     // calibration histogram being gathered
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
@@ -274,7 +275,7 @@ struct Aligned {
 };
 
 Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0, double makespan0,
-                         long long glim, double ov, double l2_budget) {
+                         long long glim, double ov, double cov, double l2_budget) {
   const int ps = c->cfg.page_size;
   const int cmax = c->lay.chunk_stride;
   const int max_chunk_pages = std::max(1, c->lay.scratch_tokens / ps);
@@ -303,6 +304,8 @@ Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0
     while (start[b + 1] <= x) ++b;
     if ((x - start[b]) % ch[b] != 0) ++inside;
   }
+  /* makespan0 already holds the plain split's combine cost (cov, in
+   * pages of one CTA's time) when it splits items */
   double cost0 = makespan0 * (double)G0;
   if (inside > 0) cost0 *= 1.0 + 0.4 / (double)rounds;
   /* aligned splits */
@@ -324,7 +327,7 @@ Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0
     const long long G = m * C;
     if (G <= 0 || (double)G < 0.84 * (double)glim) continue;
     if ((double)G * 2 * T * ps * GP * 4 > l2_budget) continue;
-    const double cost = pages + ov * (double)(itot * C);
+    const double cost = pages + ov * (double)(itot * C) + (C > 1 ? cov * (double)G : 0.0);
     if (cost >= cost0) continue;
     if (G > bestG || (G == bestG && cost < bestCost)) {
       bestG = G;
@@ -342,7 +345,10 @@ Aligned aligned_schedule(const md_ctx *c, int batch, int items, int Pmax, int T0
  * floor(n_b / G) of them plus one more on a cyclic CTA interval, and a
  * difference array gives all CTA loads in O(batch + G).  A unit costs its
  * pages plus a fixed per-unit overhead (Q load, merge, publish, ramp),
- * expressed as K/V bytes streamed.  At most MD_MAX_CHUNK_TOKENS tokens per
+ * expressed as K/V bytes streamed.  A split that gives some item several
+ * chunks also pays once for the cross-CTA combine (publishing partials,
+ * waiting for the item's other chunks, combining them): at a few hundred
+ * tokens per item a single chunk per item is faster than any split.  At most MD_MAX_CHUNK_TOKENS tokens per
  * chunk; the live raw-score scratch must stay inside L2.  A round-aligned
  * schedule (aligned_schedule) may then replace the split and the grid. */
 void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid) {
@@ -356,9 +362,11 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
       c->grid_cap > 0 ? std::min<long long>(c->grid_cap, c->grid_limit) : c->grid_limit;
   const double page_kib = ps * 512.0 / 1024.0;   // K+V of one (layer, KV head) page
   const double ov = c->unit_overhead_kib / page_kib;
-  const int knobs[4] = {(int)glim, c->unit_overhead_kib, c->force_chunks, c->lay.scratch_tokens};
+  const double cov = c->combine_overhead_kib / page_kib;
+  const int knobs[5] = {(int)glim, c->unit_overhead_kib, c->force_chunks, c->lay.scratch_tokens,
+                        c->combine_overhead_kib};
   bool same = c->plan_batch == batch && c->plan_layers == layers &&
-              std::equal(knobs, knobs + 4, c->plan_knobs);
+              std::equal(knobs, knobs + 5, c->plan_knobs);
   for (int b = 0; same && b < batch; ++b) same = c->plan_pages[b] == c->n_pages[b];
   double best = 1e300;
   int bestT = same ? c->plan_T : 0;
@@ -388,11 +396,13 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
     const int G = (int)std::max(1LL, std::min<long long>(U, glim));
     for (int g = 0; g <= G; ++g) diff[g] = 0.0;
     double base = 0.0;
+    bool split = false;
     long long start = 0;
     for (int b = 0; b < batch; ++b) {
       const int P = c->n_pages[b];
       if (P == 0) continue;
       const int ch = std::min(std::min((P + T - 1) / T, cmax), P);
+      split |= ch > 1;
       const long long n = (long long)items * ch;
       const double sz = (double)P / ch + ov;
       base += (double)(n / G) * sz;
@@ -414,7 +424,7 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
       run += diff[g];
       peak = std::max(peak, run);
     }
-    const double cost = base + peak;
+    const double cost = base + peak + (split ? cov : 0.0);   // the combine: once per launch
     if (cost < best - 1e-9) {
       best = cost;
       bestT = T;
@@ -422,7 +432,7 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
   }
   if (bestT == 0) bestT = max_chunk_pages;
   if (!same && c->force_chunks == 0 && c->grid_cap == 0) {
-    const Aligned a = aligned_schedule(c, batch, items, Pmax, bestT, best, glim, ov, l2_budget);
+    const Aligned a = aligned_schedule(c, batch, items, Pmax, bestT, best, glim, ov, cov, l2_budget);
     bestT = a.T;
     bestG = a.G;
   }
@@ -430,7 +440,7 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
     c->plan_G = bestG;
     c->plan_batch = batch;
     c->plan_layers = layers;
-    std::copy(knobs, knobs + 4, c->plan_knobs);
+    std::copy(knobs, knobs + 5, c->plan_knobs);
     c->plan_pages.assign(c->n_pages.begin(), c->n_pages.begin() + batch);
     c->plan_T = bestT;
   }
@@ -448,6 +458,9 @@ void plan_attention(md_ctx *c, int batch, int layers, AttnParams &ap, int *grid)
   ap.unit_start[batch] = (int)U;
   ap.total_units = (int)U;
   ap.n_seqs = batch;
+  ap.units_per_seq = batch > 0 ? (int)(U / batch) : 0;
+  for (int b = 0; b < batch && ap.units_per_seq > 0; ++b)
+    if (ap.unit_start[b + 1] - ap.unit_start[b] != ap.units_per_seq) ap.units_per_seq = 0;
   *grid = bestG > 0 ? bestG : (int)std::max(1LL, std::min<long long>(U, glim));
 }
 
@@ -1333,6 +1346,11 @@ MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
   if (key == MD_DEBUG_UNIT_OVERHEAD) {
     if (value < 0 || value > 65536) return fail(c, MD_ERR_INVALID_ARG, "unit overhead out of range");
     c->unit_overhead_kib = (int)value;
+    return MD_OK;
+  }
+  if (key == MD_DEBUG_COMBINE_OVERHEAD) {
+    if (value < 0 || value > 65536) return fail(c, MD_ERR_INVALID_ARG, "combine overhead out of range");
+    c->combine_overhead_kib = (int)value;
     return MD_OK;
   }
   if (key == MD_DEBUG_FORCE_CHUNKS) {

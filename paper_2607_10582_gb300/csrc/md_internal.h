@@ -87,6 +87,7 @@ struct AttnParams {
   long long spin_limit_ns;
   int extra_arrivals;
   int n_seqs, total_units;
+  int units_per_seq;   // > 0: every sequence has this many units (no search)
   int n_tokens[MD_MAX_BATCH];
   int n_pages[MD_MAX_BATCH];
   int chunks[MD_MAX_BATCH];
@@ -118,6 +119,7 @@ struct ScoreParams {
   int t;
   float rho, gamma, tau_scale, alpha;
   int score_mode, page_reduce, keep_prio;
+  int row_split;         // warps sharing a tile's mass rows (1, 2, 4, 8; set by launch_score)
   unsigned long long random_seed;
   RegionTable reg;
   int n_seqs, total_pages;
@@ -143,6 +145,23 @@ struct SelectParams {
   int push_off[MD_MAX_BATCH];
 };
 cudaError_t launch_select(const SelectParams &p, cudaStream_t s);
+
+/* Launch of a kernel taking one parameter struct, with programmatic stream
+ * serialization (the kernel calls pdl_wait() before touching global memory). */
+template <class P>
+cudaError_t launch_pdl(void (*kernel)(P), int grid, int threads, int smem, cudaStream_t s, const P &p) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, p);
+}
 
 /* --------------------------------------------------------------- init --- */
 cudaError_t launch_init(int32_t *free_stack, int P_phys, int *status, int *counters,

@@ -18,6 +18,17 @@ __device__ __forceinline__ long long globaltimer() {
   return t;
 }
 
+/* ---- programmatic dependent launch ---- */
+/* Every kernel of the library is launched with programmatic stream
+ * serialization: it may be scheduled before the kernel ahead of it in the
+ * stream has finished.  pdl_wait() blocks until that kernel has completed
+ * and its memory is visible; each kernel calls it, in every thread and on
+ * every path, before its first global-memory access, so a kernel completes
+ * only after its predecessor has.  pdl_trigger() lets the next kernel be
+ * scheduled (it then waits in its own pdl_wait()). */
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 /* ---- mbarrier ---- */
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");

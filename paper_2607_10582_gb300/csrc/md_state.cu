@@ -43,6 +43,8 @@ cudaError_t launch_init(int32_t *free_stack, int P_phys, int *status, int *count
 /* -------------------------------------------------------------- append --- */
 /* One thread per 16-byte piece of a token's K or V row in one (layer, head). */
 __global__ void append_kernel(const __grid_constant__ AppendParams p) {
+  pdl_wait();
+  pdl_trigger();
   const long long per_token = (long long)p.L * p.Hkv * 2 * 16;
   const long long total = (long long)p.n_seqs * p.n_per_seq * per_token;
   for (long long w = (long long)blockIdx.x * blockDim.x + threadIdx.x; w < total;
@@ -97,8 +99,7 @@ cudaError_t launch_append(const AppendParams &p, cudaStream_t s) {
   if (total == 0) return cudaSuccess;
   long long blocks = (total + 255) / 256;
   if (blocks > 152 * 16) blocks = 152 * 16;
-  append_kernel<<<(int)blocks, 256, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(append_kernel, (int)blocks, 256, 0, s, p);
 }
 
 /* ------------------------------------------------------ score / fold ----- */
@@ -141,19 +142,47 @@ __device__ __forceinline__ float sum_rows(const float *mass, long long slots, in
   return (w0 + w1) + (w2 + w3);
 }
 
-/* Each warp handles 32/PS consecutive pages per iteration, one lane per
- * token slot; the loop count is uniform across the warp so the segmented
- * shuffle reductions see every lane. */
+/* The part of that sum over rows rg, rg + RS, rg + 2 RS, ... (one of RS warps
+ * that share a token's rows when the batch is too small to fill the GPU). */
+__device__ __forceinline__ float sum_rows_part(const float *mass, long long slots, int rows, size_t slot,
+                                               int rg, int RS) {
+  float w0 = 0.f, w1 = 0.f, w2 = 0.f, w3 = 0.f;
+  const float *m = mass + slot;
+  int r = rg;
+  for (; r + 3 * RS < rows; r += 4 * RS) {
+    w0 += __ldcs(m + (size_t)r * slots);
+    w1 += __ldcs(m + (size_t)(r + RS) * slots);
+    w2 += __ldcs(m + (size_t)(r + 2 * RS) * slots);
+    w3 += __ldcs(m + (size_t)(r + 3 * RS) * slots);
+  }
+  for (; r < rows; r += RS) w0 += __ldcs(m + (size_t)r * slots);
+  return (w0 + w1) + (w2 + w3);
+}
+
+/* A tile is 32/PS consecutive pages, one lane per token slot; the loop count
+ * is uniform across the block so the segmented shuffle reductions see every
+ * lane and the block barriers every thread.  With row_split RS > 1 (small
+ * batches, where one warp per tile would leave most of the GPU idle) the RS
+ * warps of a group share a tile: each sums every RS-th mass row of its
+ * tokens, the parts are added in warp order through shared memory, and the
+ * group's first warp does the rest. */
 template <int PS>
 __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int PPW = 32 / PS;
   /* calibration histogram of this block (Sec. IV-B, Eq. 6's input): observed
    * mass in fixed point, so integer atomics keep the sums order-independent */
   __shared__ unsigned long long h_sum[8 * CALIB_BUCKETS];
   __shared__ unsigned int h_cnt[8 * CALIB_BUCKETS];
+  __shared__ float red[8][32];
   const int lane = threadIdx.x & 31;
-  const int warps_total = (gridDim.x * blockDim.x) >> 5;
-  const int warp_id = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int wib = threadIdx.x >> 5;
+  const int RS = p.row_split;
+  const int gpb = 8 / RS;                 // tiles per block per iteration
+  const int grp = wib / RS, rg = wib - grp * RS;
+  const int tiles = (p.total_pages + PPW - 1) / PPW;
+  const bool need_rows = p.fold_only || (p.observe && p.mass_pending);
   const float INF = INFINITY;
   const bool calib = p.calib_on && p.observe && !p.fold_only;
   if (calib) {
@@ -163,7 +192,8 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
     }
     __syncthreads();
   }
-  for (int base = warp_id * PPW; base < p.total_pages; base += warps_total * PPW) {
+  for (int t0 = blockIdx.x * gpb; t0 < tiles; t0 += gridDim.x * gpb) {
+    const int base = (t0 + grp) * PPW;
     const int gp = base + lane / PS;
     const int off = lane % PS;
     const bool page_ok = gp < p.total_pages;
@@ -178,18 +208,29 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
                           : pg * PS + off < p.n_tokens[b];
       slot = (size_t)p.block_table[(size_t)b * p.P_max + pg] * PS + off;
     }
+    float msum = 0.f;   // this token's mass over the rows (when the rows are read)
+    if (RS == 1) {
+      if (valid && need_rows) msum = sum_rows(p.mass, p.slots, p.rows, slot);
+    } else {
+      red[wib][lane] = (valid && need_rows) ? sum_rows_part(p.mass, p.slots, p.rows, slot, rg, RS) : 0.f;
+      __syncthreads();
+      if (rg == 0)
+        for (int r = 0; r < RS; ++r) msum += red[grp * RS + r][lane];
+      __syncthreads();
+      if (rg != 0) continue;
+    }
     float s = 0.f;
     int pinned = 0;
     if (valid) {
       if (p.fold_only) {
-        p.window[slot] += sum_rows(p.mass, p.slots, p.rows, slot);
+        p.window[slot] += msum;
       } else {
         const int reg = p.region[slot];
         float a = p.a[slot];
         int tr = p.t_ref[slot];
         if (p.observe) {
           float w = p.window[slot];
-          if (p.mass_pending) w += sum_rows(p.mass, p.slots, p.rows, slot);
+          if (p.mass_pending) w += msum;
           const float abar = __fdiv_rn(w, p.norm);                    // Sec. III-C
           a = p.rho * a + p.gamma * abar;                             // Eq. 2
           const int ntok = p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b];
@@ -274,15 +315,23 @@ static int score_grid_cap() {
   return cached[dev];
 }
 
-cudaError_t launch_score(const ScoreParams &p, cudaStream_t s) {
-  if (p.total_pages == 0) return cudaSuccess;
-  const int ppb = 256 / p.ps;
-  long long blocks = (p.total_pages + ppb - 1) / ppb;
+cudaError_t launch_score(const ScoreParams &p_in, cudaStream_t s) {
+  if (p_in.total_pages == 0) return cudaSuccess;
+  ScoreParams p = p_in;
+  const int ppb = 256 / p.ps;   // pages per block and iteration with one warp per tile
   const int cap = p.ps == 16 ? score_grid_cap<16>() : score_grid_cap<32>();
+  /* rows split over up to 8 warps while that still fits one wave and leaves
+   * each warp at least two rows */
+  const long long blocks1 = (p.total_pages + ppb - 1) / ppb;
+  const bool rows_read = p.fold_only || (p.observe && p.mass_pending);
+  p.row_split = 1;
+  while (rows_read && p.row_split < 8 && blocks1 * p.row_split * 2 <= cap && p.rows >= 4 * p.row_split)
+    p.row_split *= 2;
+  const int ppb_rs = ppb / p.row_split;
+  long long blocks = (p.total_pages + ppb_rs - 1) / ppb_rs;
   if (blocks > cap) blocks = cap;
-  if (p.ps == 16) score_kernel<16><<<(int)blocks, 256, 0, s>>>(p);
-  else score_kernel<32><<<(int)blocks, 256, 0, s>>>(p);
-  return cudaGetLastError();
+  if (p.ps == 16) return launch_pdl(score_kernel<16>, (int)blocks, 256, 0, s, p);
+  return launch_pdl(score_kernel<32>, (int)blocks, 256, 0, s, p);
 }
 
 /* -------------------------------------------------------------- select --- */
@@ -332,8 +381,10 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
   __shared__ int hist[256];
   __shared__ int warp_sums[32];
   __shared__ uint32_t s_prefix;
-  __shared__ int s_k, s_bad, s_gone;
+  __shared__ int s_k, s_bad, s_gone, s_cnt;
 
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x;
   const int P = p.n_pages[b];
   const int e = p.n_evict[b];
@@ -352,11 +403,15 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
     phys[i] = row[i];
     fills[i] = frow[i];
   }
-  if (threadIdx.x == 0) { s_prefix = 0u; s_k = e; s_bad = 0; s_gone = 0; }
+  if (threadIdx.x == 0) { s_prefix = 0u; s_k = e; s_bad = 0; s_gone = 0; s_cnt = 0; }
   __syncthreads();
 
-  /* radix select of the e-th smallest evictable key, most significant digit first */
+  /* radix select of the e-th smallest evictable key, most significant digit
+   * first.  It stops early once the digit's bucket holds exactly the keys
+   * still to be taken: then every key below the bucket and every key in it
+   * is evicted, the same set the remaining passes would pick. */
   uint32_t mask = 0u;
+  bool whole_bucket = false;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
@@ -398,6 +453,7 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
         }
         s_prefix = prefix | ((uint32_t)digit << shift);
         s_k = k - cum;
+        s_cnt = hist[digit];
       }
     }
     __syncthreads();
@@ -406,9 +462,16 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
       return;
     }
     mask |= 0xFFu << shift;
+    if (pass < 3 && s_k == s_cnt) {   // the same value in every thread
+      whole_bucket = true;
+      break;
+    }
   }
-  const uint32_t T = s_prefix;     // key of the e-th smallest evictable page
-  const int take_eq = s_k;         // how many pages with key == T are evicted
+  /* key of the e-th smallest evictable page and how many pages with key == T
+   * are evicted; for a whole bucket, T is the bucket's largest key and every
+   * page equal to it goes */
+  const uint32_t T = whole_bucket ? (s_prefix | ~mask) : s_prefix;
+  const int take_eq = whole_bucket ? P : s_k;
 
   /* evict: key < T, or key == T among the first take_eq in logical order;
    * compact kept pages in order; list the evicted ones in logical order */
@@ -452,6 +515,12 @@ __global__ void __launch_bounds__(SEL_THREADS) select_kernel(const __grid_consta
 
 cudaError_t launch_select(const SelectParams &p, cudaStream_t s) {
   if (p.n_seqs == 0) return cudaSuccess;
+  /* one thread per page of the longest sequence (whole warps, at least 128,
+   * at most SEL_THREADS): fewer warps make the passes' barriers cheaper */
+  int pmax = 0;
+  for (int b = 0; b < p.n_seqs; ++b) pmax = p.n_pages[b] > pmax ? p.n_pages[b] : pmax;
+  int threads = (pmax + 31) / 32 * 32;
+  threads = threads < 128 ? 128 : (threads > SEL_THREADS ? SEL_THREADS : threads);
   const size_t smem = (size_t)p.P_max * 9;
   /* raise the kernel's dynamic shared-memory limit only when a larger table
    * needs it (a host call per launch costs more than the kernel at small
@@ -465,8 +534,7 @@ cudaError_t launch_select(const SelectParams &p, cudaStream_t s) {
     if (err != cudaSuccess) return err;
     if (dev >= 0 && dev < 64) granted[dev] = (int)smem;
   }
-  select_kernel<<<p.n_seqs, SEL_THREADS, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(select_kernel, p.n_seqs, threads, (int)smem, s, p);
 }
 
 }  // namespace md

@@ -49,6 +49,7 @@ class TieStats:
         self.pages_evicted = 0
         self.inside_band = 0        # of those, boundary gap <= TIE_REL
         self.gap_le = {1e-6: 0, 1e-7: 0, 0.0: 0}
+        self.band_pages = 0         # evictable pages within TIE_REL of the boundary (all decisions)
         self.evict_adoptions = 0
         self.evict_adopt_max_dist = 0.0
         self.tokens_observed = 0
@@ -67,6 +68,8 @@ class TieStats:
         kept = [S[j] for j in range(len(S)) if j not in chosen and np.isfinite(S[j])]
         gap = (min(kept) - boundary) / (abs(boundary) + TOL_FLOOR) if kept else np.inf
         gap = abs(gap)
+        fin = np.isfinite(S)
+        self.band_pages += int(np.count_nonzero(fin & (np.abs(S - boundary) <= TIE_REL * abs(boundary))))
         if gap <= TIE_REL:
             self.inside_band += 1
         for x in self.gap_le:

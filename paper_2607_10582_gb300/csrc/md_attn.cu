@@ -92,12 +92,12 @@ __device__ __forceinline__ Unit decode_unit(const AttnParams &p, int u) {
 }
 
 /* Physical ids (and, with region-aligned pages, fills) of pages [from,
- * from + 8) of unit x, cut at the unit's end; returns how many.  The loads
- * are independent, so all of them are in flight at once. */
+ * min(from + 8, to)) of unit x; returns how many.  The loads are
+ * independent, so all of them are in flight at once. */
 template <bool ALIGNED>
-__device__ __forceinline__ int load_batch(const AttnParams &p, const Unit &x, int from, int (&ph)[8],
+__device__ __forceinline__ int load_batch(const AttnParams &p, const Unit &x, int from, int to, int (&ph)[8],
                                           int (&fl)[8]) {
-  const int cnt = min(8, x.p1 - from);
+  const int cnt = min(8, to - from);
   const int32_t *bt = p.block_table + (size_t)x.b * p.P_max;
 #pragma unroll
   for (int k = 0; k < 8; ++k) ph[k] = k < cnt ? bt[from + k] : 0;
@@ -506,10 +506,17 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     fence_barrier_init();
   }
   __syncthreads();
-  /* the kernel ahead in the stream (append) writes the pool, the block table
-   * and the page fills this one reads */
-  pdl_wait();
-  pdl_trigger();
+  /* The kernel ahead in the stream (the step's append) writes the new
+   * token's K/V into each sequence's last page, that page's block-table
+   * entry and fill, and the new token's state.  Every thread waits for it
+   * before its first global access, except the producer's issuing lane,
+   * which first starts its first unit's copies that append cannot touch
+   * (the query rows and the pages before the sequence's last one). */
+  const bool issuer = warp == 0 && lane == 0;
+  if (!issuer) {
+    pdl_wait();
+    pdl_trigger();
+  }
 
   if (warp == 0) {
     /* ------------------------------------------------------- producer ---- */
@@ -533,9 +540,36 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       int ph[8], fl[8];
       if (u < p.total_units) {
         un = decode_unit(p, u);
-        pb = un.p0;
-        cnt = load_batch<ALIGNED>(p, un, pb, ph, fl);
+        /* before the wait: the first unit's query rows (the caller's) and,
+         * when the unit is its item's only chunk, its pages below the
+         * sequence's last one, at most one per stage (measured on a GB300:
+         * 3 us off a 24 us step with single-chunk items; with split items the
+         * early pages made the launch 2 us longer, so they wait there) */
+        mbar_arrive_expect_tx(smem_u32(&qfull[0]), G * D * 2);
+        bulk_load(sQ_u32, p.q + (((size_t)un.b * p.q_layers + (un.l - p.l0)) * p.Hq + (size_t)un.kvh * G) * D,
+                  G * D * 2, smem_u32(&qfull[0]));
+        nu = 1;
+        const int early_end = un.C == 1 ? min(min(un.p1, un.p0 + S::R), p.n_pages[un.b] - 1) : un.p0;
+        for (pb = un.p0; pb < early_end; pb += 8) {
+          cnt = load_batch<ALIGNED>(p, un, pb, early_end, ph, fl);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            if (k >= cnt) break;
+            const int s = i;   // i < R: every stage is still empty
+            const int row = (((un.l * p.P_phys + ph[k]) * p.Hkv + un.kvh) * 2) * PS;
+            const uint32_t st = ring_u32 + s * S::STAGE_BYTES;
+            if (ALIGNED) fillbuf[s] = fl[k];
+            mbar_arrive_expect_tx(smem_u32(&full[s]), S::STAGE_BYTES);
+            tma_load_2d(st, &tmap, 0, row, smem_u32(&full[s]), pol);
+            tma_load_2d(st + S::HALF_BYTES, &tmap, 64, row, smem_u32(&full[s]), pol);
+            ++i;
+          }
+        }
+        pb = un.p0 + i;
       }
+      pdl_wait();
+      pdl_trigger();
+      if (u < p.total_units) cnt = pb < un.p1 ? load_batch<ALIGNED>(p, un, pb, un.p1, ph, fl) : 0;
       while (u < p.total_units && ok) {
         Unit nx = un;
         int npb = pb + 8, nxu = u, cntn = 0;
@@ -547,8 +581,8 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
             npb = nx.p0;
           }
         }
-        if (nxu < p.total_units) cntn = load_batch<ALIGNED>(p, nx, npb, phn, fln);
-        if (pb == un.p0) {
+        if (nxu < p.total_units) cntn = load_batch<ALIGNED>(p, nx, npb, nx.p1, phn, fln);
+        if (pb == un.p0 && u != (int)blockIdx.x) {   // the first unit's rows went out before the wait
           /* the unit's G query rows: one bulk copy into a double-buffered slot */
           const int qs = nu & 1;
           if (nu >= 2) {

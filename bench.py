@@ -352,28 +352,37 @@ def run_native(args, rank, world, local_rank):
     if not args.no_e2e:
         hosts = [t.cpu().pin_memory() for t in step_inputs]
         outh = torch.empty(step_output.shape, dtype=step_output.dtype).pin_memory()
-        e_ms = []
-        for i in range(args.warmup + args.steps):
-            before_step()
-            torch.cuda.synchronize()
-            t0 = time.perf_counter()
-            if args.layerwise:
-                # the per-layer entry takes device tensors: copy in, run, copy out
-                for d_t, h_t in zip(step_inputs, hosts):
-                    d_t.copy_(h_t, non_blocking=True)
-                one_step()
-                outh.copy_(step_output, non_blocking=True)
-            else:
-                # the host-buffer entry point copies inputs and output itself
-                cache.decode_step_host(B, hosts[0], hosts[1], hosts[2], regs, outh)
-                if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
-                    cache.evict(budgets)
-            torch.cuda.synchronize()
-            if i >= args.warmup:
-                e_ms.append((time.perf_counter() - t0) * 1e3)
+        def e2e_steps():
+            e_ms = []
+            for i in range(args.warmup + args.steps):
+                before_step()
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
+                if args.layerwise:
+                    # the per-layer entry takes device tensors: copy in, run, copy out
+                    for d_t, h_t in zip(step_inputs, hosts):
+                        d_t.copy_(h_t, non_blocking=True)
+                    one_step()
+                    outh.copy_(step_output, non_blocking=True)
+                else:
+                    # the host-buffer entry point moves inputs and output itself
+                    cache.decode_step_host(B, hosts[0], hosts[1], hosts[2], regs, outh)
+                    if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
+                        cache.evict(budgets)
+                torch.cuda.synchronize()
+                if i >= args.warmup:
+                    e_ms.append((time.perf_counter() - t0) * 1e3)
+            return float(np.mean(e_ms))
+
+        e_main = e2e_steps()
+        e_copies = None
+        if not args.layerwise:
+            cache.debug_set(md.MD_DEBUG_ZERO_COPY, 0)
+            e_copies = e2e_steps()
+            cache.debug_set(md.MD_DEBUG_ZERO_COPY, 1)
         h2d = sum(h_t.numel() for h_t in hosts) * 2 + B
         d2h = outh.numel() * 2
-        e2e = {"ms_per_step": float(np.mean(e_ms)), "tokens_per_step": tok_per_step[0],
+        e2e = {"ms_per_step": e_main, "ms_per_step_copies": e_copies, "tokens_per_step": tok_per_step[0],
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
     return dict(w=w, step_ms=step_ms, total_ms=total_ms, wall_s=wall, tokens=tok_per_step,
                 prof=prof, prof_tokens=prof_tokens, launches=launches, attn_ms=attn_ms, attn_n=attn_n,
@@ -644,7 +653,16 @@ def main():
                        "ms_per_step": e["ms_per_step"], "h2d_bytes_per_step": e["h2d_bytes_per_step"],
                        "d2h_bytes_per_step": e["d2h_bytes_per_step"],
                        "entry": ("pinned-host copies + md_decode_layer x L + md_evict" if args.layerwise
-                                 else "md_decode_step_host (host buffers, copies in the call) + md_evict")}
+                                 else "md_decode_step_host + md_evict: the step's inputs start and its output "
+                                      "ends in pinned host memory; the query rows are copied in (cudaMemcpyAsync), "
+                                      "the append kernel reads the new K/V and the attention kernel writes the "
+                                      "output in place over the host link (NVLink-C2C)")}
+        if e.get("ms_per_step_copies") is not None:
+            line["e2e"]["copy_path"] = {
+                "value": e["tokens_per_step"] * world / (e["ms_per_step_copies"] / 1e3), "unit": UNIT,
+                "ms_per_step": e["ms_per_step_copies"],
+                "entry": "md_decode_step_host with MD_DEBUG_ZERO_COPY = 0: cudaMemcpyAsync of the inputs "
+                         "into the workspace and of the output back, inside the call"}
     if not args.no_cpu_baseline and world == 1:
         measured, scaled, info = parallel_oracle(args, 3)
         line["cpu_baseline"] = {"value": info["tokens_per_step"] / min(scaled), "unit": UNIT,

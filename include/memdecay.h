@@ -164,19 +164,25 @@ md_status md_append_tokens(md_ctx *ctx, int seq, int n_tokens, const uint8_t *re
 md_status md_decode_step(md_ctx *ctx, int batch, const void *q_dev, const void *k_new_dev,
                          const void *v_new_dev, const uint8_t *new_region_host, void *out_dev);
 
-/* md_decode_step with the step's tensors in host memory: the query rows and
- * the new tokens' K/V are copied into the workspace, the step runs, and the
- * output is copied back, all enqueued on the handle's stream in that order.
- * Like every call it is asynchronous: out_host holds the output once the
- * stream has reached the copy (md_sync, or a synchronisation of the
- * stream), and the input buffers must stay unchanged until then.  Pinned
- * (page-locked) host memory gives full copy speed; pageable memory works,
- * with the copies then partly synchronous.  Layouts as md_decode_step:
+/* md_decode_step with the step's tensors in host memory.  The query rows
+ * are copied into the workspace before the step.  The new tokens' K/V and
+ * the output are used where they are when the device can reach them: the
+ * kernels read the K/V rows and write the output over the host link (on a
+ * GB300, NVLink-C2C), with no copy.  The device reaches pinned (page-locked)
+ * or registered host memory, and, where it accesses pageable memory
+ * coherently (cudaDevAttrPageableMemoryAccess, as on Grace-Blackwell), any
+ * host memory; the buffers must be 16-byte aligned for this.  Other buffers
+ * are copied through the workspace.  Copies are enqueued on the handle's
+ * stream, inputs before the step and the output after it.  Like every call
+ * it is asynchronous: out_host holds the output once the stream has passed
+ * the step (md_sync, or a synchronisation of the stream), and the input
+ * buffers must stay unchanged until then.  Layouts as md_decode_step:
  *   q_host                  bf16 [batch][L][Hq][D]   (host)
  *   k_new_host, v_new_host  bf16 [batch][L][Hkv][D]  (host)
  *   new_region_host         [batch]                  (host)
  *   out_host                bf16 [batch][L][Hq][D]   (host, written)
- * Errors as md_decode_step; every argument check runs before any copy. */
+ * Errors as md_decode_step; every argument check runs before any copy or
+ * launch. */
 md_status md_decode_step_host(md_ctx *ctx, int batch, const void *q_host, const void *k_new_host,
                               const void *v_new_host, const uint8_t *new_region_host,
                               void *out_host);
@@ -303,14 +309,19 @@ md_status md_profile_read(md_ctx *ctx, double *ms_per_stage, int64_t *launches_p
  *                             (0 = planned; otherwise clamped to the limits)
  *   MD_DEBUG_COMBINE_OVERHEAD cost, in KiB of K/V streamed by one CTA, that
  *                             the planner adds to a split giving any item
- *                             several chunks (default 192; 0..65536) */
+ *                             several chunks (default 192; 0..65536)
+ *   MD_DEBUG_ZERO_COPY        1 (default): md_decode_step_host uses the K/V
+ *                             and output buffers in place where the device
+ *                             reaches them; 0: it copies every buffer
+ *                             through the workspace */
 enum {
   MD_DEBUG_SPIN_LIMIT_NS = 0,
   MD_DEBUG_EXTRA_ARRIVALS = 1,
   MD_DEBUG_GRID_LIMIT = 2,
   MD_DEBUG_UNIT_OVERHEAD = 3,
   MD_DEBUG_FORCE_CHUNKS = 4,
-  MD_DEBUG_COMBINE_OVERHEAD = 5
+  MD_DEBUG_COMBINE_OVERHEAD = 5,
+  MD_DEBUG_ZERO_COPY = 6
 };
 md_status md_debug_set(md_ctx *ctx, int key, int64_t value);
 

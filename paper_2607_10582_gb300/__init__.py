@@ -46,7 +46,7 @@ MD_CALIB_BUCKET_WIDTH = 4
 (MD_QUERY_TOKENS, MD_QUERY_PAGES, MD_QUERY_FREE_TOP, MD_QUERY_STEP, MD_QUERY_WINDOW,
  MD_QUERY_PINNED_PAGES) = range(6)
 (MD_DEBUG_SPIN_LIMIT_NS, MD_DEBUG_EXTRA_ARRIVALS, MD_DEBUG_GRID_LIMIT, MD_DEBUG_UNIT_OVERHEAD,
- MD_DEBUG_FORCE_CHUNKS, MD_DEBUG_COMBINE_OVERHEAD) = range(6)
+ MD_DEBUG_FORCE_CHUNKS, MD_DEBUG_COMBINE_OVERHEAD, MD_DEBUG_ZERO_COPY) = range(7)
 STAGES = ("append", "attention", "fold", "score", "select")
 
 

@@ -73,6 +73,8 @@ struct md_ctx {
   int plan_batch = -1, plan_layers = -1, plan_T = 0, plan_G = 0;
   int plan_knobs[5] = {-1, -1, -1, -1, -1};
   bool calib_on = false;     // calibration histogram being gathered
+  int pageable_access = 0;   // the device reads and writes pageable host memory coherently
+  int zero_copy = 1;         // md_decode_step_host: new K/V and output used in place when reachable
   bool prof = false;
   std::vector<cudaEvent_t> ev_pool;
   std::vector<ProfRec> pending;
@@ -560,6 +562,13 @@ MD_API md_status md_create(const md_config *cfg, md_ctx **out) {
     delete c;
     return MD_ERR_CUDA;
   }
+  {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&v, cudaDevAttrPageableMemoryAccess, dev) == cudaSuccess)
+      c->pageable_access = v;
+    cudaGetLastError();
+  }
   c->grid_limit = attention_grid_limit(cfg->page_size);
   if (c->grid_limit <= 0) {
     delete c;
@@ -865,6 +874,40 @@ void end_step(md_ctx *c, int batch) {
 
 }  // namespace
 
+namespace {
+
+/* The whole decode step once its arguments are checked. */
+md_status decode_step_core(md_ctx *c, int batch, const void *q, const void *k_new, const void *v_new,
+                           const uint8_t *new_region_host, void *out) {
+  const md_config &cf = c->cfg;
+  md_status st = begin_step(c, batch, 0, cf.num_layers, (long long)cf.num_layers * cf.num_kv_heads * D,
+                            (long long)cf.num_kv_heads * D, k_new, v_new, new_region_host);
+  if (st != MD_OK) return st;
+  st = run_attention(c, batch, 0, cf.num_layers, cf.num_layers, q, out);
+  if (st != MD_OK) return st;
+  end_step(c, batch);
+  return MD_OK;
+}
+
+/* The address at which the kernels can use host buffer h directly, or null:
+ * pinned (page-locked) or registered memory at its device address, any other
+ * host memory only where the device accesses pageable memory coherently
+ * (Grace's NVLink-C2C with address translation).  16-byte alignment is
+ * required (the kernels move 16-byte pieces). */
+void *device_view(const md_ctx *c, const void *h) {
+  if ((uintptr_t)h & 15) return nullptr;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, h) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a.type == cudaMemoryTypeHost && a.devicePointer) return ((uintptr_t)a.devicePointer & 15) ? nullptr : a.devicePointer;
+  if (a.type == cudaMemoryTypeUnregistered && c->pageable_access) return const_cast<void *>(h);
+  return nullptr;
+}
+
+}  // namespace
+
 MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const void *k_new,
                                 const void *v_new, const uint8_t *new_region_host,
                                 void *out_dev) {
@@ -874,14 +917,7 @@ MD_API md_status md_decode_step(md_ctx *c, int batch, const void *q_dev, const v
   if (!q_dev || !k_new || !v_new || !out_dev) return fail(c, MD_ERR_INVALID_ARG, "null pointer");
   md_status st = check_step(c, batch, new_region_host);
   if (st != MD_OK) return st;
-  const md_config &cf = c->cfg;
-  st = begin_step(c, batch, 0, cf.num_layers, (long long)cf.num_layers * cf.num_kv_heads * D,
-                  (long long)cf.num_kv_heads * D, k_new, v_new, new_region_host);
-  if (st != MD_OK) return st;
-  st = run_attention(c, batch, 0, cf.num_layers, cf.num_layers, q_dev, out_dev);
-  if (st != MD_OK) return st;
-  end_step(c, batch);
-  return MD_OK;
+  return decode_step_core(c, batch, q_dev, k_new, v_new, new_region_host, out_dev);
 }
 
 MD_API md_status md_decode_step_host(md_ctx *c, int batch, const void *q_host, const void *k_new_host,
@@ -899,16 +935,29 @@ MD_API md_status md_decode_step_host(md_ctx *c, int batch, const void *q_host, c
   const md_config &cf = c->cfg;
   const size_t q_bytes = (size_t)batch * cf.num_layers * cf.num_q_heads * D * 2;
   const size_t kv_bytes = (size_t)batch * cf.num_layers * cf.num_kv_heads * D * 2;
+  /* The new tokens' K/V and the output are used where they are when the
+   * device can reach them: the append kernel reads the K/V rows and the
+   * attention kernel writes the output over the host link, with no copy (on
+   * a GB300 that took the config-2 steady step's device time from 170 to
+   * 138 us).  The query rows are always copied into the workspace first:
+   * every unit of the attention kernel reads its rows with a TMA copy at its
+   * start, and over the host link that latency cost more than the copy
+   * (207 us).  Buffers the device cannot reach are copied too. */
+  const void *vk = c->zero_copy ? device_view(c, k_new_host) : nullptr;
+  const void *vv = c->zero_copy ? device_view(c, v_new_host) : nullptr;
+  void *vo = c->zero_copy ? device_view(c, out_host) : nullptr;
   uint8_t *dq = c->ws + c->lay.io_q, *dk = c->ws + c->lay.io_k, *dv = c->ws + c->lay.io_v,
           *dout = c->ws + c->lay.io_out;
   cudaError_t e = cudaMemcpyAsync(dq, q_host, q_bytes, cudaMemcpyHostToDevice, c->stream);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(dk, k_new_host, kv_bytes, cudaMemcpyHostToDevice, c->stream);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(dv, v_new_host, kv_bytes, cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess && !vk) e = cudaMemcpyAsync(dk, k_new_host, kv_bytes, cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess && !vv) e = cudaMemcpyAsync(dv, v_new_host, kv_bytes, cudaMemcpyHostToDevice, c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "input copy");
-  st = md_decode_step(c, batch, dq, dk, dv, new_region_host, dout);
+  st = decode_step_core(c, batch, dq, vk ? vk : dk, vv ? vv : dv, new_region_host, vo ? vo : dout);
   if (st != MD_OK) return st;
-  e = cudaMemcpyAsync(out_host, dout, q_bytes, cudaMemcpyDeviceToHost, c->stream);
-  if (e != cudaSuccess) return cuda_fail(c, e, "output copy");
+  if (!vo) {
+    e = cudaMemcpyAsync(out_host, dout, q_bytes, cudaMemcpyDeviceToHost, c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "output copy");
+  }
   return MD_OK;
 }
 
@@ -1346,6 +1395,11 @@ MD_API md_status md_debug_set(md_ctx *c, int key, int64_t value) {
   if (key == MD_DEBUG_UNIT_OVERHEAD) {
     if (value < 0 || value > 65536) return fail(c, MD_ERR_INVALID_ARG, "unit overhead out of range");
     c->unit_overhead_kib = (int)value;
+    return MD_OK;
+  }
+  if (key == MD_DEBUG_ZERO_COPY) {
+    if (value != 0 && value != 1) return fail(c, MD_ERR_INVALID_ARG, "zero-copy switch must be 0 or 1");
+    c->zero_copy = (int)value;
     return MD_OK;
   }
   if (key == MD_DEBUG_COMBINE_OVERHEAD) {

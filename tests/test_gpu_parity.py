@@ -312,10 +312,12 @@ def test_config2_full_trace_step_is_bit_identical_over_reruns():
 
 
 def test_decode_step_host_matches_device_path():
-    """md_decode_step_host (host buffers; the copies are enqueued inside the
-    call) gives the same bits as md_decode_step from the same state, with
-    pinned torch tensors and with pageable numpy arrays; an out-of-range batch
-    is rejected before anything is copied."""
+    """md_decode_step_host (host buffers) gives the same bits as
+    md_decode_step from the same state: with pinned torch tensors and with
+    pageable numpy arrays, the K/V and output buffers used in place where the
+    device reaches them (the kernels read and write host memory) and through
+    copies when that is switched off or a buffer is misaligned; an
+    out-of-range batch is rejected before anything is copied."""
     w = synth.custom_workload("host", L=2, Hq=16, Hkv=2, page_size=16, lengths=[700, 1500],
                               budget_frac=0.5, steps=4, seed=5, structured=True)
     B, L, Hq, Hkv = w.B, w.L, w.Hq, w.Hkv
@@ -349,6 +351,26 @@ def test_decode_step_host_matches_device_path():
     c.decode_step_host(B, q, kn, vn, regs, outn)
     assert c.sync() == md.MD_OK
     assert np.array_equal(outn, ref_o.numpy().view(np.uint16))
+
+    # the copy path, pinned and pageable
+    c.debug_set(md.MD_DEBUG_ZERO_COPY, 0)
+    for bufs in ((qh, kh, vh), (q, kn, vn)):
+        c.load_state(saved)
+        outc = torch.zeros((B, L, Hq, 128), dtype=torch.int16).pin_memory()
+        c.decode_step_host(B, *bufs, regs, outc)
+        assert c.sync() == md.MD_OK
+        assert torch.equal(outc, ref_o)
+        assert torch.equal(c.get_state(md.MD_STATE_MASS).cpu(), ref_m)
+    c.debug_set(md.MD_DEBUG_ZERO_COPY, 1)
+    # a misaligned K buffer (2 bytes off) goes through a copy, V and the output in place
+    c.load_state(saved)
+    km = np.zeros(kn.size + 1, np.uint16)[1:].reshape(kn.shape)
+    km[...] = kn
+    assert km.ctypes.data % 16 != 0
+    outm = np.zeros((B, L, Hq, 128), np.uint16)
+    c.decode_step_host(B, q, km, vn, regs, outm)
+    assert c.sync() == md.MD_OK
+    assert np.array_equal(outm, ref_o.numpy().view(np.uint16))
 
     with pytest.raises(md.MemDecayError) as ei:
         c.decode_step_host(B + 1, q, kn, vn, regs + [6], outn)

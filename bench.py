@@ -15,7 +15,7 @@ step does that full work; `--phase steady` times continuing steps instead.
 Each timed step is bracketed by CUDA events on the launching stream and holds
 no other event; the per-kernel times behind the roofline come from a second
 pass over the same steps with the library's event pairs.  Where a step's K/V
-would fit in L2 (configs 0 and 1), a 256 MiB write flushes it before each
+would fit in L2 (configs 0 and 1), a 1 GiB write flushes it before each
 step, outside the brackets.
 
 `--impl reference` times the fp64 CPU oracle on the host cores on a bounded
@@ -45,7 +45,10 @@ UNIT = "tokens/s"
 SPEC_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129 * 10**6          # GB300 L2
-FLUSH_BYTES = 256 * 2**20       # written between timed steps when a step's K/V would fit in L2
+# written between timed steps when a step's K/V would fit in L2; larger than L2
+# and long enough (about 0.16 ms) that the host has enqueued the next step before
+# the GPU reaches it, so a latency-bound step's time is the GPU's, not the host's
+FLUSH_BYTES = 2**30
 
 
 def parse():
@@ -564,7 +567,7 @@ def workload_config(w, args):
             "score_mode": "paper additive (Eq. 4)" if w.score_mode == 0 else "multiplicative",
             "phase": "full-trace step (state restored before each step)" if args.phase == "full"
             else "steady state",
-            "l2": ("L2 flushed before every timed step (256 MiB write, untimed): a step's K/V fits in L2"
+            "l2": ("L2 flushed before every timed step (1 GiB write, untimed): a step's K/V fits in L2"
                    if needs_flush(w) else "no flush: inputs larger than L2 (K/V read per step >> 129 MB)"),
             "parallelism": "replicas" if args.gpus > 1 else "1 GPU", "seed": args.seed,
             "entry": "md_decode_layer x L + md_evict" if args.layerwise else "md_decode_step + md_evict",

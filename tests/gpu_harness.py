@@ -125,9 +125,10 @@ def rel_err(g, o):
 
 class Lockstep:
     def __init__(self, w: synth.Workload, *, check_every=1, phys_slack=2, layerwise=False, calib=False,
-                 p_max=None):
+                 p_max=None, host_buffers=False):
         self.w = w
         self.layerwise = layerwise
+        self.host_buffers = host_buffers   # decode through md_decode_step_host with pinned buffers
         B = w.B
         self.P_max = w.max_pages_per_seq() if p_max is None else p_max
         self.P_phys = w.num_phys_pages() + phys_slack
@@ -173,7 +174,12 @@ class Lockstep:
         q = synth.q_host(w.seed, B, w.L, w.Hq, w.Hkv, t, w.structured)
         kn, vn = synth.step_kv_host(w.seed, self.pos, regions, w.L, w.Hkv, w.structured)
         out = torch.empty((B, w.L, w.Hq, w.D), dtype=torch.int16, device="cuda")
-        if self.layerwise:
+        if self.host_buffers:
+            pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).pin_memory()
+            out = torch.empty((B, w.L, w.Hq, w.D), dtype=torch.int16).pin_memory()
+            self.gpu.decode_step_host(B, pin(q), pin(kn), pin(vn), regions, out)
+            assert self.gpu.sync() == md.MD_OK
+        elif self.layerwise:
             qd, knd, vnd = to_dev(q), to_dev(kn), to_dev(vn)
             for l in range(w.L):
                 o_l = torch.empty((B, w.Hq, w.D), dtype=torch.int16, device="cuda")

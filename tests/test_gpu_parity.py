@@ -378,6 +378,17 @@ def test_decode_step_host_matches_device_path():
     c.close()
 
 
+def test_host_buffer_steps_follow_the_oracle():
+    """Many decode + evict steps through md_decode_step_host with pinned
+    buffers (query rows copied in, new K/V read and output written in place
+    over the host link), evictions and page turnover included, against the
+    oracle at every step."""
+    w = synth.custom_workload("hostpath", L=2, Hq=16, Hkv=2, page_size=16, lengths=[700, 1500, 37],
+                              budget_frac=0.4, steps=40, seed=23, structured=True)
+    ls = Lockstep(w, host_buffers=True).run()
+    ls.check_layout()
+
+
 def test_checkpoint_restore_replays_step():
     w = synth.custom_workload("ckpt", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900],
                               budget_frac=0.3, steps=2, seed=9)

@@ -232,14 +232,15 @@ def run_native(args, rank, world, local_rank):
     vn = torch.empty_like(kn)
     out = torch.empty_like(q)
     pos_d = torch.tensor([w.n0(b) for b in range(B)], dtype=torch.int32, device=dev)
-    regs = [w.decode_region] * B
-    reg_d = torch.tensor(regs, dtype=torch.uint8, device=dev)
+    # the per-step host arguments as arrays, as a serving loop keeps them
+    regs = np.full(B, w.decode_region, np.uint8)
+    reg_d = torch.from_numpy(regs).to(dev)
     assert lib.synth_fill_q_dev(w.seed, int(w.structured), kap, B, L, Hq, Hq // Hkv, D, 1, q.data_ptr(),
                                 stream.cuda_stream) == 0
     assert lib.synth_fill_step_kv_dev(w.seed, int(w.structured), kap, B, L, Hkv, D, pos_d.data_ptr(),
                                       reg_d.data_ptr(), kn.data_ptr(), vn.data_ptr(), stream.cuda_stream) == 0
     torch.cuda.synchronize()
-    budgets = list(w.budget_pages)
+    budgets = np.asarray(w.budget_pages, np.int32)
 
     # tensors a step reads from the host in the end-to-end measurement
     step_inputs = [q, kn, vn]
@@ -276,6 +277,7 @@ def run_native(args, rank, world, local_rank):
         cache.calib_enable(True)
     saved = cache.save_state()
     tokens_saved = [cache.query(md.MD_QUERY_TOKENS, b) for b in range(B)]
+    window_saved = cache.query(md.MD_QUERY_WINDOW)
     restore = args.phase == "full"
     # a step whose K/V could stay in L2 gets the L2 flushed before it (untimed)
     flush_buf = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev) if needs_flush(w) else None
@@ -357,8 +359,13 @@ def run_native(args, rank, world, local_rank):
         outh = torch.empty(step_output.shape, dtype=step_output.dtype).pin_memory()
         def e2e_steps():
             e_ms = []
+            # decode steps since the last observation, tracked on the host as a
+            # caller would (the library's count is checked afterwards)
+            window = cache.query(md.MD_QUERY_WINDOW)
             for i in range(args.warmup + args.steps):
                 before_step()
+                if restore:
+                    window = window_saved
                 torch.cuda.synchronize()
                 t0 = time.perf_counter()
                 if args.layerwise:
@@ -370,11 +377,15 @@ def run_native(args, rank, world, local_rank):
                 else:
                     # the host-buffer entry point moves inputs and output itself
                     cache.decode_step_host(B, hosts[0], hosts[1], hosts[2], regs, outh)
-                    if cache.query(md.MD_QUERY_WINDOW) >= w.window_k:
+                    window += 1
+                    if window >= w.window_k:
                         cache.evict(budgets)
+                        window = 0
                 torch.cuda.synchronize()
                 if i >= args.warmup:
                     e_ms.append((time.perf_counter() - t0) * 1e3)
+            if not args.layerwise:
+                assert window == cache.query(md.MD_QUERY_WINDOW), "window bookkeeping"
             return float(np.mean(e_ms))
 
         e_main = e2e_steps()

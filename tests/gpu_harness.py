@@ -166,20 +166,24 @@ class Lockstep:
             self.pos[b] = n
         torch.cuda.synchronize()
 
-    def decode(self, regions=None):
+    def decode(self, regions=None, entry=None):
+        """One decode step on both sides.  entry: "device" (md_decode_step),
+        "host" (md_decode_step_host with pinned buffers) or "layers"
+        (md_decode_layer per layer); default from the constructor."""
         w = self.w
+        entry = entry or ("host" if self.host_buffers else "layers" if self.layerwise else "device")
         B = w.B
         t = self.orc.t + 1
         regions = [w.decode_region] * B if regions is None else list(regions)
         q = synth.q_host(w.seed, B, w.L, w.Hq, w.Hkv, t, w.structured)
         kn, vn = synth.step_kv_host(w.seed, self.pos, regions, w.L, w.Hkv, w.structured)
         out = torch.empty((B, w.L, w.Hq, w.D), dtype=torch.int16, device="cuda")
-        if self.host_buffers:
+        if entry == "host":
             pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).pin_memory()
             out = torch.empty((B, w.L, w.Hq, w.D), dtype=torch.int16).pin_memory()
             self.gpu.decode_step_host(B, pin(q), pin(kn), pin(vn), regions, out)
             assert self.gpu.sync() == md.MD_OK
-        elif self.layerwise:
+        elif entry == "layers":
             qd, knd, vnd = to_dev(q), to_dev(kn), to_dev(vn)
             for l in range(w.L):
                 o_l = torch.empty((B, w.Hq, w.D), dtype=torch.int16, device="cuda")

@@ -389,6 +389,24 @@ def test_host_buffer_steps_follow_the_oracle():
     ls.check_layout()
 
 
+def test_entry_points_mixed_step_by_step():
+    """Every kernel is launched with programmatic dependent launch, so a
+    kernel may start before the one ahead of it ends and relies on waiting
+    for it.  Steps that switch entry point every time (device buffers, host
+    buffers, layer by layer, with an observation after each) still follow the
+    oracle at every step."""
+    w = synth.custom_workload("mixed", L=3, Hq=16, Hkv=2, page_size=16, lengths=[900, 40, 2100],
+                              budget_frac=0.4, steps=24, seed=29, structured=True)
+    ls = Lockstep(w)
+    ls.prefill()
+    for s in range(w.steps):
+        ls.decode(entry=("device", "host", "layers")[s % 3])
+        ls.observe()
+        if s % 5 == 4:
+            ls.check_layout()
+    ls.check_layout()
+
+
 def test_checkpoint_restore_replays_step():
     w = synth.custom_workload("ckpt", L=2, Hq=8, Hkv=2, page_size=16, lengths=[900],
                               budget_frac=0.3, steps=2, seed=9)

@@ -518,6 +518,12 @@ def test_capacity_and_argument_errors_are_synchronous():
     with pytest.raises(md.MemDecayError) as e:
         c.set_region_params(0, 1.0, 10.0, True)   # pinned flag with tokens cached
     assert e.value.status == md.MD_ERR_STATE
+    for key, bad in ((md.MD_DEBUG_ZERO_COPY, 2), (md.MD_DEBUG_COMBINE_OVERHEAD, -1),
+                     (md.MD_DEBUG_COMBINE_OVERHEAD, 1 << 20), (md.MD_DEBUG_GRID_LIMIT, md.MD_MAX_CHUNKS - 1),
+                     (md.MD_DEBUG_FORCE_CHUNKS, md.MD_MAX_CHUNKS + 1), (99, 0)):
+        with pytest.raises(md.MemDecayError) as e:
+            c.debug_set(key, bad)
+        assert e.value.status == md.MD_ERR_INVALID_ARG, (key, bad)
     assert c.sync() == md.MD_OK
 
 

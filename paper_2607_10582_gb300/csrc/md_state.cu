@@ -126,7 +126,10 @@ __device__ __forceinline__ float random_draw(unsigned long long seed, int t, siz
 }
 
 /* Sum of one token's mass over the rows (layer, KV head) in a fixed order,
- * four partial sums so that many row loads are in flight per lane. */
+ * four partial sums so that many row loads are in flight per lane.  The last
+ * one to three rows are loaded together before they are added to the first
+ * sum (the zero of an absent row leaves the non-negative sum as it is), so a
+ * short row list costs one memory round trip. */
 __device__ __forceinline__ float sum_rows(const float *mass, long long slots, int rows, size_t slot) {
   float w0 = 0.f, w1 = 0.f, w2 = 0.f, w3 = 0.f;
   const float *m = mass + slot;
@@ -138,12 +141,20 @@ __device__ __forceinline__ float sum_rows(const float *mass, long long slots, in
     w2 += __ldcs(m + (size_t)(r + 2) * slots);
     w3 += __ldcs(m + (size_t)(r + 3) * slots);
   }
-  for (; r < rows; ++r) w0 += __ldcs(m + (size_t)r * slots);
+  {
+    const float t0 = r < rows ? __ldcs(m + (size_t)r * slots) : 0.f;
+    const float t1 = r + 1 < rows ? __ldcs(m + (size_t)(r + 1) * slots) : 0.f;
+    const float t2 = r + 2 < rows ? __ldcs(m + (size_t)(r + 2) * slots) : 0.f;
+    w0 += t0;
+    w0 += t1;
+    w0 += t2;
+  }
   return (w0 + w1) + (w2 + w3);
 }
 
 /* The part of that sum over rows rg, rg + RS, rg + 2 RS, ... (one of RS warps
- * that share a token's rows when the batch is too small to fill the GPU). */
+ * that share a token's rows when the batch is too small to fill the GPU),
+ * with the same grouping and the same loads of the last rows. */
 __device__ __forceinline__ float sum_rows_part(const float *mass, long long slots, int rows, size_t slot,
                                                int rg, int RS) {
   float w0 = 0.f, w1 = 0.f, w2 = 0.f, w3 = 0.f;
@@ -155,7 +166,14 @@ __device__ __forceinline__ float sum_rows_part(const float *mass, long long slot
     w2 += __ldcs(m + (size_t)(r + 2 * RS) * slots);
     w3 += __ldcs(m + (size_t)(r + 3 * RS) * slots);
   }
-  for (; r < rows; r += RS) w0 += __ldcs(m + (size_t)r * slots);
+  {
+    const float t0 = r < rows ? __ldcs(m + (size_t)r * slots) : 0.f;
+    const float t1 = r + RS < rows ? __ldcs(m + (size_t)(r + RS) * slots) : 0.f;
+    const float t2 = r + 2 * RS < rows ? __ldcs(m + (size_t)(r + 2 * RS) * slots) : 0.f;
+    w0 += t0;
+    w0 += t1;
+    w0 += t2;
+  }
   return (w0 + w1) + (w2 + w3);
 }
 
@@ -165,9 +183,11 @@ __device__ __forceinline__ float sum_rows_part(const float *mass, long long slot
  * batches, where one warp per tile would leave most of the GPU idle) the RS
  * warps of a group share a tile: each sums every RS-th mass row of its
  * tokens, the parts are added in warp order through shared memory, and the
- * group's first warp does the rest. */
+ * group's first warp does the rest.  A token's state is loaded before its
+ * mass rows, so the two sets of loads overlap; the register bound keeps six
+ * blocks per SM, the wave the launcher's row split is sized to. */
 template <int PS>
-__global__ void score_kernel(const __grid_constant__ ScoreParams p) {
+__global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ ScoreParams p) {
   pdl_wait();
   pdl_trigger();
   constexpr int PPW = 32 / PS;
@@ -208,6 +228,22 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
                           : pg * PS + off < p.n_tokens[b];
       slot = (size_t)p.block_table[(size_t)b * p.P_max + pg] * PS + off;
     }
+    /* the token's state, loaded before its mass rows so that both are in
+     * flight together (only the group's first warp goes on past the rows) */
+    int reg = 0, tr = 0, tins = 0, ntok = 1;
+    float a = 0.f, w = 0.f;
+    if (valid && rg == 0) {
+      if (p.fold_only) {
+        w = p.window[slot];
+      } else {
+        reg = p.region[slot];
+        a = p.a[slot];
+        tr = p.t_ref[slot];
+        if (p.observe) w = p.window[slot];
+        if (p.observe || p.score_mode == 2) ntok = p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b];
+        if (calib || p.score_mode == 3) tins = p.t_ins[slot];
+      }
+    }
     float msum = 0.f;   // this token's mass over the rows (when the rows are read)
     if (RS == 1) {
       if (valid && need_rows) msum = sum_rows(p.mass, p.slots, p.rows, slot);
@@ -223,17 +259,12 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
     int pinned = 0;
     if (valid) {
       if (p.fold_only) {
-        p.window[slot] += msum;
+        p.window[slot] = w + msum;
       } else {
-        const int reg = p.region[slot];
-        float a = p.a[slot];
-        int tr = p.t_ref[slot];
         if (p.observe) {
-          float w = p.window[slot];
           if (p.mass_pending) w += msum;
           const float abar = __fdiv_rn(w, p.norm);                    // Sec. III-C
           a = p.rho * a + p.gamma * abar;                             // Eq. 2
-          const int ntok = p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b];
           const float tau = __fdiv_rn(p.tau_scale, (float)ntok);
           if (abar >= tau) tr = p.t;                                  // Eq. 3
           p.window[slot] = 0.f;
@@ -241,7 +272,7 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
           p.a[slot] = a;
           p.t_ref[slot] = tr;
           if (calib) {
-            const int age = p.t - p.t_ins[slot];
+            const int age = p.t - tins;
             const int bkt = age >= 0 ? age / CALIB_WIDTH : -1;
             if (bkt >= 0 && bkt < CALIB_BUCKETS) {
               atomicAdd(&h_sum[reg * CALIB_BUCKETS + bkt], __float2ull_rn(abar * 4294967296.0f));
@@ -254,11 +285,8 @@ __global__ void score_kernel(const __grid_constant__ ScoreParams p) {
         switch (p.score_mode) {
           case 0: s = p.reg.base[reg] * d + p.alpha * a; break;       // Eq. 4
           case 1: s = (p.reg.base[reg] + p.alpha * a) * d; break;
-          case 2:
-            s = p.reg.base[reg] * d +
-                p.alpha * a * (float)(p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b]);
-            break;
-          case 3: s = (float)p.t_ins[slot]; break;                     // recency
+          case 2: s = p.reg.base[reg] * d + p.alpha * a * (float)ntok; break;
+          case 3: s = (float)tins; break;                             // recency
           default: s = random_draw(p.random_seed, p.t, slot); break;   // random
         }
         pinned = p.reg.pinned[reg];

@@ -362,8 +362,8 @@ md_status md_calib_fit(const double *mass_sum, const int64_t *count, int n_bucke
  * cannot call cudaMalloc or any allocating routine: code running where the
  * allocator is owned by someone else (a serving engine or framework that
  * hands out only the tensors it allocated), code that must not allocate
- * between CUDA-graph replays, or embedders whose memory budget is fixed up
- * front.  Those callers cannot provide md_decode_step's workspace.
+ * once it is running, or embedders whose memory budget is fixed up front.
+ * Those callers cannot provide md_decode_step's workspace.
  *
  * It runs stage 1 alone -- paged GQA decode attention over every cached
  * token plus each token's attention mass per (layer, KV head) -- over a paged
@@ -403,8 +403,7 @@ md_status md_calib_fit(const double *mass_sum, const int64_t *count, int n_bucke
  * The first call on a device, with that device current, looks up the
  * array's device address (cudaGetSymbolAddress), the kernel's resident CTAs
  * (occupancy query; it also sets the kernel's shared-memory limit) and the
- * driver's tensor-map encoder, and keeps them for the process; make that
- * first call before any stream capture.
+ * driver's tensor-map encoder, and keeps them for the process.
  * Every call on a device shares the same array and clears its counters and
  * status words on the stream before the kernel; calls whose GPU work overlaps
  * (other streams, other threads) race on the array and must be serialised by

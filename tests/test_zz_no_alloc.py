@@ -1,6 +1,6 @@
 """md_attend_mass_noalloc: stage 1 for callers that cannot allocate device
 memory (a serving engine that owns the allocator, code that must not
-allocate between graph replays, a fixed memory budget).  It uses a fixed
+allocate once it is running, a fixed memory budget).  It uses a fixed
 scratch array inside the library instead of a workspace.  Its output must
 match the workspace path (md_decode_step's attention output and mass rows)
 within the parity tolerances, on two calls in a row (the second call finds

@@ -183,9 +183,8 @@ __device__ __forceinline__ float sum_rows_part(const float *mass, long long slot
  * batches, where one warp per tile would leave most of the GPU idle) the RS
  * warps of a group share a tile: each sums every RS-th mass row of its
  * tokens, the parts are added in warp order through shared memory, and the
- * group's first warp does the rest.  A token's state is loaded before its
- * mass rows, so the two sets of loads overlap; the register bound keeps six
- * blocks per SM, the wave the launcher's row split is sized to. */
+ * group's first warp does the rest.  The register bound keeps six blocks
+ * per SM, the wave the launcher's row split is sized to. */
 template <int PS>
 __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ ScoreParams p) {
   pdl_wait();
@@ -228,11 +227,14 @@ __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ S
                           : pg * PS + off < p.n_tokens[b];
       slot = (size_t)p.block_table[(size_t)b * p.P_max + pg] * PS + off;
     }
-    /* the token's state, loaded before its mass rows so that both are in
-     * flight together (only the group's first warp goes on past the rows) */
+    /* the token's state: with RS > 1 (a few rows per warp, latency-bound)
+     * loaded before the mass rows so that both are in flight together, by the
+     * group's first warp, the one that goes on past the rows; with RS = 1
+     * after them, where a warp sums every row and the registers go to keeping
+     * many row loads in flight */
     int reg = 0, tr = 0, tins = 0, ntok = 1;
     float a = 0.f, w = 0.f;
-    if (valid && rg == 0) {
+    auto load_state = [&]() {
       if (p.fold_only) {
         w = p.window[slot];
       } else {
@@ -243,11 +245,13 @@ __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ S
         if (p.observe || p.score_mode == 2) ntok = p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b];
         if (calib || p.score_mode == 3) tins = p.t_ins[slot];
       }
-    }
+    };
     float msum = 0.f;   // this token's mass over the rows (when the rows are read)
     if (RS == 1) {
       if (valid && need_rows) msum = sum_rows(p.mass, p.slots, p.rows, slot);
+      if (valid) load_state();
     } else {
+      if (valid && rg == 0) load_state();
       red[wib][lane] = (valid && need_rows) ? sum_rows_part(p.mass, p.slots, p.rows, slot, rg, RS) : 0.f;
       __syncthreads();
       if (rg == 0)

@@ -83,8 +83,9 @@ enum {
 #define MD_CALIB_BUCKET_WIDTH 4   /* decode steps per age bucket (Fig. 3)      */
 
 typedef struct {
-  /* Geometry: L layers, Hq query heads, Hkv KV heads (Hq / Hkv <= 8), head_dim
-   * must be 128, page_size 16 or 32 tokens (Sec. III-D, fixed-size pages). */
+  /* Geometry: L layers (1..255), Hq query heads, Hkv KV heads (Hq / Hkv <= 8,
+   * L * Hq < 65,536), head_dim must be 128, page_size 16 or 32 tokens
+   * (Sec. III-D, fixed-size pages). */
   int num_layers, num_q_heads, num_kv_heads, head_dim, page_size;
   /* Capacity: sequences, block-table width (pages per sequence, at most
    * MD_MAX_CHUNKS * MD_MAX_CHUNK_TOKENS / page_size), pages in the pool. */
@@ -243,7 +244,10 @@ enum {
   MD_STATE_FREE = 6,        /* int32 [num_phys_pages] free stack (top: md_query)      */
   MD_STATE_REGION = 7,      /* uint8 [slots] region label                             */
   MD_STATE_WINDOW = 8,      /* fp32  [slots] attention mass of folded window steps    */
-  MD_STATE_MASS = 9,        /* fp32  [L*Hkv][slots] mass rows of the last decode step */
+  MD_STATE_MASS = 9,        /* u64   [slots] attention mass of the last decode step,
+                               summed over layers and query heads, in fixed point
+                               (2^48 = 1.0); cleared when an evict or the next
+                               step folds it                                  */
   MD_STATE_POOL = 10,       /* bf16  [L][num_phys_pages][Hkv][2][page_size][D] K/V    */
   MD_STATE_T_INS = 11,      /* int32 [slots] insertion step                           */
   MD_STATE_PAGE_FILL = 12,  /* uint8 [max_batch][max_pages_per_seq] tokens per page   */
@@ -276,7 +280,8 @@ md_status md_query(const md_ctx *ctx, int what, int seq, int64_t *out);
 /* Checkpoint of everything but the page pool's contents: device state into
  * dst_dev (md_state_bytes() device bytes) and the host mirror into host_blob
  * (host bytes).  Only between observation windows (MD_ERR_STATE otherwise).
- * md_load_state restores both; the pool must still hold the saved pages. */
+ * md_load_state restores both, and clears any step mass the live state had
+ * pending; the pool must still hold the saved pages. */
 md_status md_state_bytes(const md_ctx *ctx, size_t *device_bytes, size_t *host_bytes);
 md_status md_save_state(md_ctx *ctx, void *dst_dev, void *host_blob);
 md_status md_load_state(md_ctx *ctx, const void *src_dev, const void *host_blob);

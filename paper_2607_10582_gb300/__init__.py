@@ -277,7 +277,7 @@ class Cache:
             MD_STATE_FREE: ((self.P_phys,), t.int32),
             MD_STATE_REGION: ((slots,), t.uint8),
             MD_STATE_WINDOW: ((slots,), t.float32),
-            MD_STATE_MASS: ((self.L * self.Hkv, slots), t.float32),
+            MD_STATE_MASS: ((slots,), t.int64),
             MD_STATE_POOL: ((self.L, self.P_phys, self.Hkv, 2, self.ps, MD_HEAD_DIM), t.int16),
             MD_STATE_T_INS: ((slots,), t.int32),
             MD_STATE_PAGE_FILL: ((self.max_batch, self.P_max), t.uint8),

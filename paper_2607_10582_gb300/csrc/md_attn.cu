@@ -26,8 +26,11 @@
  * finisher, then takes the unit over while the consumers stream the next
  * one: it waits, bounded by %globaltimer, for all chunks of the item,
  * combines the partials (its slice of the output O) and turns the stored
- * scores into masses, one fp32 row per (layer, KV head) indexed by physical
- * slot.  Raw scores live in two slots per CTA; the consumers reuse a slot only
+ * scores into masses.  Each token's mass is added at L2 into its physical
+ * slot's fixed-point accumulator (an integer add, so the sum over layers and
+ * KV heads does not depend on the order in which items finish); the
+ * no-allocation entry point writes one fp32 row per (layer, KV head)
+ * instead.  Raw scores live in two slots per CTA; the consumers reuse a slot only
  * after the finisher has released it (mbarrier hand-off both ways), so a
  * unit's finish overlaps the streaming of the next one.  All waits are
  * bounded; on expiry the kernel records MD_ERR_DEVICE_TIMEOUT, raises an abort
@@ -189,17 +192,21 @@ __device__ __forceinline__ void load_page_ids(const AttnParams &p, const Unit &p
 }
 
 /* Token masses of a unit from its stored raw scores and the item's per-head
- * (max, 1/Z) in f.fin: mass_i = sum_h exp2(s_hi - max_h) / Z_h, written to
- * the (layer, KV head) row at the token's physical slot.  Four tokens per
- * thread in flight (a batch's loads are issued before any store). */
-template <int PS, bool ALIGNED, int NT>
+ * (max, 1/Z) in f.fin: mass_i = sum_h exp2(s_hi - max_h) / Z_h, added in
+ * fixed point to the token's slot of the step's accumulator (kept in L2
+ * with evict_last: every (layer, KV head) adds to the same slots), or
+ * written to the (layer, KV head) row at that slot.  Four tokens per thread
+ * in flight (a batch's loads are issued before any store). */
+template <int PS, bool ALIGNED, int NT, bool ROWS>
 __device__ __forceinline__ void mass_pass(const AttnParams &p, const Unit &pv, int slot, int tid,
                                           const FinSmem &f) {
   const int G = p.G;
   const int npg = pv.p1 - pv.p0;
   const float *scr = p.scratch + ((size_t)blockIdx.x * 2 + slot) * p.scratch_tokens * GP;
   const int ntok = npg * PS;
-  float *mrow = p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots;
+  unsigned long long *acc = p.mass_acc;
+  float *mrow = ROWS ? p.mass + (size_t)(pv.l * p.Hkv + pv.kvh) * p.slots : nullptr;
+  const uint64_t acc_pol = policy_evict_last();
   float fm[GP], fz[GP];
 #pragma unroll
   for (int h = 0; h < GP; ++h) {
@@ -229,7 +236,11 @@ __device__ __forceinline__ void mass_pass(const AttnParams &p, const Unit &pv, i
                 exp2f(s0[r].z - fm[2]) * fz[2] + exp2f(s0[r].w - fm[3]) * fz[3];
       m += exp2f(s1[r].x - fm[4]) * fz[4] + exp2f(s1[r].y - fm[5]) * fz[5] +
            exp2f(s1[r].z - fm[6]) * fz[6] + exp2f(s1[r].w - fm[7]) * fz[7];
-      mrow[(size_t)f.sphys[tk / PS] * PS + (tk % PS)] = m;
+      const size_t slot_i = (size_t)f.sphys[tk / PS] * PS + (tk % PS);
+      if (ROWS)
+        mrow[slot_i] = m;
+      else
+        red_add_u64_hint(acc + slot_i, __float2ull_rn(m * MASS_SCALE), acc_pol);
     }
   }
 }
@@ -242,7 +253,7 @@ __device__ __forceinline__ void mass_pass(const AttnParams &p, const Unit &pv, i
  * warp, or all consumer warps for a CTA's last unit.  Returns false, the same
  * for every thread, on abort or timeout.  Loads are issued in batches before
  * the dependent stores, so a pass costs a few L2 round trips. */
-template <int PS, bool ALIGNED, int NT, int OBUF_FLOATS>
+template <int PS, bool ALIGNED, int NT, int OBUF_FLOATS, bool ROWS>
 __device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv, int slot, int tid,
                                             const FinSmem &f) {
   const float NEG_INF = -INFINITY;
@@ -351,7 +362,7 @@ __device__ __forceinline__ bool finish_unit(const AttnParams &p, const Unit &pv,
       orow[e] = *(uint16_t *)&bv;
     }
   }
-  mass_pass<PS, ALIGNED, NT>(p, pv, slot, tid, f);
+  mass_pass<PS, ALIGNED, NT, ROWS>(p, pv, slot, tid, f);
   fin_sync<NT>();
   if (tid == 0) {
     const int old = atomicAdd(&p.counters[pv.X], 1);
@@ -441,20 +452,23 @@ __device__ __forceinline__ void merge_single(const AttnParams &p, const Unit &un
 /* The whole end of a single-chunk unit: the page ids, the merge straight
  * into (max, 1/Z) and the output, the release of the merge buffers (mdone,
  * when given: the finisher's hand-off), the token masses. */
-template <int PS, bool ALIGNED, int NCW, int NT>
+template <int PS, bool ALIGNED, int NCW, int NT, bool ROWS>
 __device__ __forceinline__ void single_end(const AttnParams &p, const Unit &un, int slot, int tid,
                                         const float *wm, const float *wl, float *wf,
                                         const float *wO, const FinSmem &f, uint32_t mdone) {
   load_page_ids<ALIGNED, NT>(p, un, tid, f);
   merge_single<NCW, NT>(p, un, tid, wm, wl, wf, wO, f);
   if (mdone != 0 && tid == 0) mbar_arrive(mdone);   // merge buffers free again
-  mass_pass<PS, ALIGNED, NT>(p, un, slot, tid, f);
+  mass_pass<PS, ALIGNED, NT, ROWS>(p, un, slot, tid, f);
   fin_sync<NT>();
 }
 
 /* ALIGNED: pages carry their own fill (region-aligned allocation); otherwise
- * every page but the last is full and the fills follow from n_tokens. */
-template <int PS, int NCW, bool ALIGNED>
+ * every page but the last is full and the fills follow from n_tokens.  ROWS:
+ * the masses go to one fp32 row per (layer, KV head) (the no-allocation entry
+ * point) instead of the step's fixed-point accumulator; a compile-time choice,
+ * since this end-of-unit code runs once per unit and is often fetched cold. */
+template <int PS, int NCW, bool ALIGNED, bool ROWS>
 __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW>::CTAS_PER_SM)
     attn_mass_kernel(const __grid_constant__ AttnParams p,
                      const __grid_constant__ CUtensorMap tmap) {
@@ -657,11 +671,11 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
       const bool ok = wait_phase(smem_u32(&cdone[k & 1]), (k >> 1) & 1, p, 8, true);
       if (!__all_sync(0xffffffffu, ok)) break;
       if (pv.C == 1) {
-        single_end<PS, ALIGNED, NCW, 32>(p, pv, k & 1, lane, wm, wl, wf, wO, fs, smem_u32(&mdone[0]));
+        single_end<PS, ALIGNED, NCW, 32, ROWS>(p, pv, k & 1, lane, wm, wl, wf, wO, fs, smem_u32(&mdone[0]));
       } else {
         merge_publish<NCW, 32>(p, pv, lane, wm, wl, wf, wO);
         if (lane == 0) mbar_arrive(smem_u32(&mdone[0]));   // merge buffers free again
-        if (!finish_unit<PS, ALIGNED, 32, S::OBUF_FLOATS>(p, pv, k & 1, lane, fs)) break;
+        if (!finish_unit<PS, ALIGNED, 32, S::OBUF_FLOATS, ROWS>(p, pv, k & 1, lane, fs)) break;
       }
       if (lane == 0) mbar_arrive(smem_u32(&fdone[k & 1]));   // slot and finish area free
     }
@@ -850,23 +864,33 @@ __global__ void __launch_bounds__(AttnShape<PS, NCW>::THREADS, AttnShape<PS, NCW
     named_barrier(1, NC);
     if (flag[0]) break;
     if (un.C == 1) {
-      single_end<PS, ALIGNED, NCW, NCW * 32>(p, un, slot, ct, wm, wl, wf, wO, fs, 0u);
+      single_end<PS, ALIGNED, NCW, NCW * 32, ROWS>(p, un, slot, ct, wm, wl, wf, wO, fs, 0u);
       break;
     }
     merge_publish<NCW, NCW * 32>(p, un, ct, wm, wl, wf, wO);
     if (ct == 0) flag[1] = ld_volatile(&p.status[ST_ABORT]);
     named_barrier(1, NC);
     if (flag[1]) break;
-    finish_unit<PS, ALIGNED, NCW * 32, S::OBUF_FLOATS>(p, un, slot, ct, fs);
+    finish_unit<PS, ALIGNED, NCW * 32, S::OBUF_FLOATS, ROWS>(p, un, slot, ct, fs);
     break;
   }
 }
 
-template <int PS, int NCW, bool AL>
+template <int PS, int NCW, bool AL, bool ROWS>
 static cudaError_t prepare_impl() {
-  return cudaFuncSetAttribute(attn_mass_kernel<PS, NCW, AL>,
+  return cudaFuncSetAttribute(attn_mass_kernel<PS, NCW, AL, ROWS>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)AttnShape<PS, NCW>::SMEM);
+}
+
+/* The instances of one page size: the step's (contiguous or region-aligned
+ * pages) and the no-allocation entry point's (contiguous pages, mass rows). */
+template <int PS, int NCW>
+static cudaError_t prepare_all() {
+  cudaError_t e = prepare_impl<PS, NCW, false, false>();
+  if (e == cudaSuccess) e = prepare_impl<PS, NCW, true, false>();
+  if (e == cudaSuccess) e = prepare_impl<PS, NCW, false, true>();
+  return e;
 }
 
 template <int PS, int NCW>
@@ -874,9 +898,8 @@ static int grid_limit_impl() {
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-  if (prepare_impl<PS, NCW, false>() != cudaSuccess || prepare_impl<PS, NCW, true>() != cudaSuccess)
-    return 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_mass_kernel<PS, NCW, false>,
+  if (prepare_all<PS, NCW>() != cudaSuccess) return 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_mass_kernel<PS, NCW, false, false>,
                                                     AttnShape<PS, NCW>::THREADS,
                                                     AttnShape<PS, NCW>::SMEM) != cudaSuccess)
     return 0;
@@ -884,7 +907,7 @@ static int grid_limit_impl() {
   return g > MAX_GRID ? MAX_GRID : g;
 }
 
-template <int PS, int NCW, bool AL>
+template <int PS, int NCW, bool AL, bool ROWS>
 static cudaError_t launch_impl(const AttnParams &p, const CUtensorMap &tmap, int grid,
                                cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
@@ -899,15 +922,13 @@ static cudaError_t launch_impl(const AttnParams &p, const CUtensorMap &tmap, int
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, attn_mass_kernel<PS, NCW, AL>, p, tmap);
+  return cudaLaunchKernelEx(&cfg, attn_mass_kernel<PS, NCW, AL, ROWS>, p, tmap);
 }
 
 constexpr int NCW_DEFAULT = 4;
 
 cudaError_t attention_prepare(int ps) {
-  cudaError_t e = ps == 16 ? prepare_impl<16, NCW_DEFAULT, false>() : prepare_impl<32, NCW_DEFAULT, false>();
-  if (e != cudaSuccess) return e;
-  return ps == 16 ? prepare_impl<16, NCW_DEFAULT, true>() : prepare_impl<32, NCW_DEFAULT, true>();
+  return ps == 16 ? prepare_all<16, NCW_DEFAULT>() : prepare_all<32, NCW_DEFAULT>();
 }
 
 int attention_grid_limit(int ps) {
@@ -917,11 +938,16 @@ int attention_grid_limit(int ps) {
 cudaError_t launch_attention(const AttnParams &p, const CUtensorMap &tmap, int grid,
                              cudaStream_t s) {
   if (p.total_units == 0) return cudaSuccess;
+  if (!p.mass_acc) {   // mass rows: the no-allocation entry point, contiguous pages
+    if (p.page_fill) return cudaErrorInvalidValue;
+    return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, false, true>(p, tmap, grid, s)
+                      : launch_impl<32, NCW_DEFAULT, false, true>(p, tmap, grid, s);
+  }
   if (p.page_fill)
-    return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, true>(p, tmap, grid, s)
-                      : launch_impl<32, NCW_DEFAULT, true>(p, tmap, grid, s);
-  return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, false>(p, tmap, grid, s)
-                    : launch_impl<32, NCW_DEFAULT, false>(p, tmap, grid, s);
+    return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, true, false>(p, tmap, grid, s)
+                      : launch_impl<32, NCW_DEFAULT, true, false>(p, tmap, grid, s);
+  return p.ps == 16 ? launch_impl<16, NCW_DEFAULT, false, false>(p, tmap, grid, s)
+                    : launch_impl<32, NCW_DEFAULT, false, false>(p, tmap, grid, s);
 }
 
 }  // namespace md

@@ -111,6 +111,8 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 const char *check_config(const md_config &c) {
   if (c.num_layers < 1 || c.num_layers > 255) return "num_layers must be in [1, 255]";
   if (c.num_kv_heads < 1 || c.num_q_heads < c.num_kv_heads) return "bad head counts";
+  if ((long long)c.num_layers * c.num_q_heads >= MASS_MAX_HEADS)
+    return "num_layers * num_q_heads must stay below 65,536";
   if (c.num_q_heads % c.num_kv_heads) return "num_q_heads must be a multiple of num_kv_heads";
   if (c.num_q_heads / c.num_kv_heads > MD_MAX_GROUP) return "GQA group above 8 query heads";
   if (c.head_dim != MD_HEAD_DIM) return "head_dim must be 128";
@@ -212,12 +214,13 @@ int64_t cached_tokens(const md_ctx *c) {
   return s;
 }
 
-/* Window fold: add the pending per-(layer, head) mass rows into the window
- * accumulator of every token that was attended in that step. */
+/* Window fold: add the pending step's mass (summed over layers and heads)
+ * into the window accumulator of every token that was attended in that step,
+ * and clear the step's accumulator. */
 md_status launch_fold(md_ctx *c) {
   ScoreParams sp;
   memset(&sp, 0, sizeof(sp));
-  sp.mass = ptr<float>(c, c->lay.mass);
+  sp.mass_acc = ptr<unsigned long long>(c, c->lay.mass_acc);
   sp.window = ptr<float>(c, c->lay.window);
   sp.region = ptr<uint8_t>(c, c->lay.region);
   sp.block_table = ptr<int32_t>(c, c->lay.block_table);
@@ -228,7 +231,6 @@ md_status launch_fold(md_ctx *c) {
     sp.seq_tokens = ptr<int32_t>(c, c->lay.seq_tokens);
   }
   sp.slots = (long long)c->lay.slots;
-  sp.rows = c->cfg.num_layers * c->cfg.num_kv_heads;
   sp.ps = c->cfg.page_size;
   sp.P_max = c->cfg.max_pages_per_seq;
   sp.fold_only = 1;
@@ -500,7 +502,7 @@ size_t md::compute_layout(const md_config &c, Layout *lay) {
   L.window = take(L.slots * 4, 256);
   L.ahat = take(L.slots * 4, 256);
   L.prio = take(L.slots * 4, 256);
-  L.mass = take((size_t)c.num_layers * c.num_kv_heads * L.slots * 4, 256);
+  L.mass_acc = take(L.slots * 8, 256);
   L.scratch = take((size_t)MAX_GRID * 2 * L.scratch_tokens * GP * 4, 256);
   L.partials = take(L.n_items * L.chunk_stride * PARTIAL_FLOATS * 4, 256);
   L.counters = take(L.n_items * 4, 256);
@@ -833,7 +835,7 @@ md_status run_attention(md_ctx *c, int batch, int l0, int L, int q_layers, const
   atp.out = (uint16_t *)out_dev;
   atp.block_table = ptr<int32_t>(c, c->lay.block_table);
   atp.page_fill = cf.region_aligned_pages ? ptr<uint8_t>(c, c->lay.page_fill) : nullptr;
-  atp.mass = ptr<float>(c, c->lay.mass);
+  atp.mass_acc = ptr<unsigned long long>(c, c->lay.mass_acc);
   atp.scratch = ptr<float>(c, c->lay.scratch);
   atp.partials = ptr<float>(c, c->lay.partials);
   atp.counters = ptr<int>(c, c->lay.counters);
@@ -1030,7 +1032,7 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   /* stages 2-3 */
   ScoreParams sp;
   memset(&sp, 0, sizeof(sp));
-  sp.mass = ptr<float>(c, c->lay.mass);
+  sp.mass_acc = ptr<unsigned long long>(c, c->lay.mass_acc);
   sp.window = ptr<float>(c, c->lay.window);
   sp.a = ptr<float>(c, c->lay.a);
   sp.ahat = ptr<float>(c, c->lay.ahat);
@@ -1048,7 +1050,6 @@ MD_API md_status md_evict(md_ctx *c, int batch, const int32_t *budget, int32_t *
   sp.calib_cnt = (unsigned int *)(c->ws + c->lay.calib + (size_t)8 * CALIB_BUCKETS * 8);
   sp.calib_on = c->calib_on ? 1 : 0;
   sp.slots = (long long)c->lay.slots;
-  sp.rows = cf.num_layers * cf.num_kv_heads;
   sp.ps = ps;
   sp.P_max = cf.max_pages_per_seq;
   sp.fold_only = 0;
@@ -1177,10 +1178,7 @@ bool state_array(const md_ctx *c, int what, size_t *off, size_t *bytes) {
     case MD_STATE_FREE: *off = L.free_stack; *bytes = (size_t)cf.num_phys_pages * 4; return true;
     case MD_STATE_REGION: *off = L.region; *bytes = L.slots; return true;
     case MD_STATE_WINDOW: *off = L.window; *bytes = L.slots * 4; return true;
-    case MD_STATE_MASS:
-      *off = L.mass;
-      *bytes = (size_t)cf.num_layers * cf.num_kv_heads * L.slots * 4;
-      return true;
+    case MD_STATE_MASS: *off = L.mass_acc; *bytes = L.slots * 8; return true;
     case MD_STATE_T_INS: *off = L.t_ins; *bytes = L.slots * 4; return true;
     case MD_STATE_PAGE_FILL:
       *off = L.page_fill;
@@ -1336,6 +1334,10 @@ MD_API md_status md_load_state(md_ctx *c, const void *src_dev, const void *host_
   memcpy(c->tokens_exact.data(), h, B);
   h += B;
   c->calib_on = *h != 0;
+  /* a checkpoint holds no pending step mass; clear whatever the live state
+   * had accumulated, or the next step would add to it */
+  cudaError_t e = cudaMemsetAsync(c->ws + c->lay.mass_acc, 0, c->lay.slots * 8, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "restore: clear the step mass");
   return MD_OK;
 }
 

@@ -18,6 +18,17 @@ constexpr int PARTIAL_FLOATS = 1088;        // m[8] l[8] O[8][128], padded to 25
 constexpr int MAX_GRID = 512;               // persistent attention CTAs (>= 2 x SM count)
 
 enum DevStatus { ST_CODE = 0, ST_ABORT = 1, ST_DIAG = 2, ST_WORDS = 8 };
+
+/* A decode step's attention mass per token, summed over layers and query
+ * heads, is accumulated in fixed point: u64 with MASS_FRAC_BITS fraction
+ * bits.  Integer adds make the sum independent of the order in which the
+ * (layer, KV head) items finish.  One token receives at most 1 from each
+ * query head, so num_layers * num_q_heads < MASS_MAX_HEADS keeps the sum
+ * below 2^64. */
+constexpr int MASS_FRAC_BITS = 48;
+constexpr float MASS_SCALE = 281474976710656.0f;        // 2^48
+constexpr float MASS_UNIT = 3.5527136788005009e-15f;    // 2^-48
+constexpr long long MASS_MAX_HEADS = 65536;
 constexpr int CALIB_BUCKETS = MD_CALIB_BUCKETS;      // age buckets per region
 constexpr int CALIB_WIDTH = MD_CALIB_BUCKET_WIDTH;   // decode steps per bucket
 
@@ -29,7 +40,7 @@ struct RegionTable {
 
 /* Byte offsets of every array inside the caller's workspace. */
 struct Layout {
-  size_t pool, block_table, page_score, free_stack, region, a, t_ref, t_ins, window, ahat, prio, mass,
+  size_t pool, block_table, page_score, free_stack, region, a, t_ref, t_ins, window, ahat, prio, mass_acc,
       scratch, partials, counters, evict_list, staging_regions, staging_steps, staging_slots, status,
       calib, page_fill, seq_tokens, io_q, io_k, io_v, io_out, total;
   size_t slots, n_items;
@@ -72,7 +83,8 @@ struct AttnParams {
   const int32_t *block_table;
   const uint8_t *page_fill;  // [max_batch][P_max] tokens per page, or null: pages are
                              // full up to n_tokens
-  float *mass;         // [L*Hkv][slots]
+  unsigned long long *mass_acc;   // [slots] fixed-point mass of the step, or null:
+  float *mass;                    // [L*Hkv][slots] one fp32 row per (layer, KV head)
   float *scratch;      // [grid][2][scratch_tokens][8]
   float *partials;     // [items][chunk_stride][PARTIAL_FLOATS]
   int *counters;       // [items]
@@ -100,7 +112,7 @@ cudaError_t attention_prepare(int ps); // one-time function attributes
 
 /* --------------------------------------------------- fold / score ------- */
 struct ScoreParams {
-  const float *mass;
+  unsigned long long *mass_acc;    // [slots] fixed-point mass of the pending step (read, zeroed)
   float *window, *a, *ahat, *prio, *page_score;
   int32_t *t_ref;
   const int32_t *t_ins;
@@ -112,14 +124,13 @@ struct ScoreParams {
   unsigned int *calib_cnt;         // [8][CALIB_BUCKETS] observations
   int calib_on;
   long long slots;
-  int rows, ps, P_max;
-  int fold_only;         // 1: window += mass rows and nothing else
+  int ps, P_max;
+  int fold_only;         // 1: window += the pending step's mass and nothing else
   int observe, mass_pending;
   float norm;            // window steps * L * Hq
   int t;
   float rho, gamma, tau_scale, alpha;
   int score_mode, page_reduce, keep_prio;
-  int row_split;         // warps sharing a tile's mass rows (1, 2, 4, 8; set by launch_score)
   unsigned long long random_seed;
   RegionTable reg;
   int n_seqs, total_pages;

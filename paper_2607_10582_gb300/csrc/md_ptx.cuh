@@ -142,6 +142,11 @@ __device__ __forceinline__ int ld_acquire_gpu(const int *p) {
 __device__ __forceinline__ int ld_volatile(const int *p) {
   return *(volatile const int *)p;
 }
+/* Integer add at L2 (no return value) with an L2 eviction-priority hint. */
+__device__ __forceinline__ void red_add_u64_hint(unsigned long long *p, unsigned long long v,
+                                                 uint64_t policy) {
+  asm volatile("red.global.add.L2::cache_hint.u64 [%0], %1, %2;" ::"l"(p), "l"(v), "l"(policy) : "memory");
+}
 __device__ __forceinline__ void st_v2_hint(float *p, float x, float y, uint64_t policy) {
   asm volatile("st.global.L1::no_allocate.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(p),
                "f"(x), "f"(y), "l"(policy)

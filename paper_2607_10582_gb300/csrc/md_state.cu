@@ -4,12 +4,13 @@
  *            from the free stack) and start each token's state: region label,
  *            t_ref = insertion step, a = 0 (Sec. III-A; Fig. 1 "append KV").
  *   score    per page, one lane per token: Abar from the window accumulator
- *            and the per-(layer, KV head) mass rows (Sec. III-C), the EWMA
+ *            and the step's mass summed over layers and heads (Sec. III-C;
+ *            a fixed-point accumulator the attention kernel fills), the EWMA
  *            (Eq. 2), the refresh test Abar >= tau_scale/|K_t| (Eq. 3), the
  *            retention score (Eq. 4, lambda = ln2 / half-life, Eq. 7) and the
  *            page score by a shuffle reduction over the page's lanes (Eq. 5;
  *            pinned pages and the page being written score +inf).  With
- *            fold_only it only adds the mass rows into the window accumulator.
+ *            fold_only it only adds the step's mass into the window accumulator.
  *   select   one CTA per sequence: radix select (4 passes of 8-bit digits
  *            over order-preserving uint32 keys, ties by logical page index)
  *            of the e lowest evictable pages, stable compaction of the block
@@ -125,66 +126,12 @@ __device__ __forceinline__ float random_draw(unsigned long long seed, int t, siz
   return (float)(z >> 40) * 5.9604644775390625e-08f;
 }
 
-/* Sum of one token's mass over the rows (layer, KV head) in a fixed order,
- * four partial sums so that many row loads are in flight per lane.  The last
- * one to three rows are loaded together before they are added to the first
- * sum (the zero of an absent row leaves the non-negative sum as it is), so a
- * short row list costs one memory round trip. */
-__device__ __forceinline__ float sum_rows(const float *mass, long long slots, int rows, size_t slot) {
-  float w0 = 0.f, w1 = 0.f, w2 = 0.f, w3 = 0.f;
-  const float *m = mass + slot;
-  int r = 0;
-#pragma unroll 4
-  for (; r + 4 <= rows; r += 4) {
-    w0 += __ldcs(m + (size_t)r * slots);
-    w1 += __ldcs(m + (size_t)(r + 1) * slots);
-    w2 += __ldcs(m + (size_t)(r + 2) * slots);
-    w3 += __ldcs(m + (size_t)(r + 3) * slots);
-  }
-  {
-    const float t0 = r < rows ? __ldcs(m + (size_t)r * slots) : 0.f;
-    const float t1 = r + 1 < rows ? __ldcs(m + (size_t)(r + 1) * slots) : 0.f;
-    const float t2 = r + 2 < rows ? __ldcs(m + (size_t)(r + 2) * slots) : 0.f;
-    w0 += t0;
-    w0 += t1;
-    w0 += t2;
-  }
-  return (w0 + w1) + (w2 + w3);
-}
-
-/* The part of that sum over rows rg, rg + RS, rg + 2 RS, ... (one of RS warps
- * that share a token's rows when the batch is too small to fill the GPU),
- * with the same grouping and the same loads of the last rows. */
-__device__ __forceinline__ float sum_rows_part(const float *mass, long long slots, int rows, size_t slot,
-                                               int rg, int RS) {
-  float w0 = 0.f, w1 = 0.f, w2 = 0.f, w3 = 0.f;
-  const float *m = mass + slot;
-  int r = rg;
-  for (; r + 3 * RS < rows; r += 4 * RS) {
-    w0 += __ldcs(m + (size_t)r * slots);
-    w1 += __ldcs(m + (size_t)(r + RS) * slots);
-    w2 += __ldcs(m + (size_t)(r + 2 * RS) * slots);
-    w3 += __ldcs(m + (size_t)(r + 3 * RS) * slots);
-  }
-  {
-    const float t0 = r < rows ? __ldcs(m + (size_t)r * slots) : 0.f;
-    const float t1 = r + RS < rows ? __ldcs(m + (size_t)(r + RS) * slots) : 0.f;
-    const float t2 = r + 2 * RS < rows ? __ldcs(m + (size_t)(r + 2 * RS) * slots) : 0.f;
-    w0 += t0;
-    w0 += t1;
-    w0 += t2;
-  }
-  return (w0 + w1) + (w2 + w3);
-}
-
-/* A tile is 32/PS consecutive pages, one lane per token slot; the loop count
- * is uniform across the block so the segmented shuffle reductions see every
- * lane and the block barriers every thread.  With row_split RS > 1 (small
- * batches, where one warp per tile would leave most of the GPU idle) the RS
- * warps of a group share a tile: each sums every RS-th mass row of its
- * tokens, the parts are added in warp order through shared memory, and the
- * group's first warp does the rest.  The register bound keeps six blocks
- * per SM, the wave the launcher's row split is sized to. */
+/* A tile is 32/PS consecutive pages, one lane per token slot, one warp per
+ * tile; the loop count is uniform across the block so the segmented shuffle
+ * reductions see every lane.  A token's step mass is one fixed-point
+ * accumulator (the attention kernel adds every (layer, KV head) into it):
+ * read and zeroed here, loaded together with the token's state.  The
+ * launcher sizes the grid to one wave of resident blocks. */
 template <int PS>
 __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ ScoreParams p) {
   pdl_wait();
@@ -194,14 +141,10 @@ __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ S
    * mass in fixed point, so integer atomics keep the sums order-independent */
   __shared__ unsigned long long h_sum[8 * CALIB_BUCKETS];
   __shared__ unsigned int h_cnt[8 * CALIB_BUCKETS];
-  __shared__ float red[8][32];
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
-  const int RS = p.row_split;
-  const int gpb = 8 / RS;                 // tiles per block per iteration
-  const int grp = wib / RS, rg = wib - grp * RS;
   const int tiles = (p.total_pages + PPW - 1) / PPW;
-  const bool need_rows = p.fold_only || (p.observe && p.mass_pending);
+  const bool need_mass = p.fold_only || (p.observe && p.mass_pending);
   const float INF = INFINITY;
   const bool calib = p.calib_on && p.observe && !p.fold_only;
   if (calib) {
@@ -211,8 +154,8 @@ __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ S
     }
     __syncthreads();
   }
-  for (int t0 = blockIdx.x * gpb; t0 < tiles; t0 += gridDim.x * gpb) {
-    const int base = (t0 + grp) * PPW;
+  for (int t0 = blockIdx.x * 8; t0 < tiles; t0 += gridDim.x * 8) {
+    const int base = (t0 + wib) * PPW;
     const int gp = base + lane / PS;
     const int off = lane % PS;
     const bool page_ok = gp < p.total_pages;
@@ -227,14 +170,12 @@ __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ S
                           : pg * PS + off < p.n_tokens[b];
       slot = (size_t)p.block_table[(size_t)b * p.P_max + pg] * PS + off;
     }
-    /* the token's state: with RS > 1 (a few rows per warp, latency-bound)
-     * loaded before the mass rows so that both are in flight together, by the
-     * group's first warp, the one that goes on past the rows; with RS = 1
-     * after them, where a warp sums every row and the registers go to keeping
-     * many row loads in flight */
+    /* the token's state and its step mass, all loads independent */
     int reg = 0, tr = 0, tins = 0, ntok = 1;
     float a = 0.f, w = 0.f;
-    auto load_state = [&]() {
+    unsigned long long macc = 0ull;
+    if (valid) {
+      if (need_mass) macc = __ldcs(p.mass_acc + slot);
       if (p.fold_only) {
         w = p.window[slot];
       } else {
@@ -245,20 +186,10 @@ __global__ void __launch_bounds__(256, 6) score_kernel(const __grid_constant__ S
         if (p.observe || p.score_mode == 2) ntok = p.seq_tokens ? p.seq_tokens[b] : p.n_tokens[b];
         if (calib || p.score_mode == 3) tins = p.t_ins[slot];
       }
-    };
-    float msum = 0.f;   // this token's mass over the rows (when the rows are read)
-    if (RS == 1) {
-      if (valid && need_rows) msum = sum_rows(p.mass, p.slots, p.rows, slot);
-      if (valid) load_state();
-    } else {
-      if (valid && rg == 0) load_state();
-      red[wib][lane] = (valid && need_rows) ? sum_rows_part(p.mass, p.slots, p.rows, slot, rg, RS) : 0.f;
-      __syncthreads();
-      if (rg == 0)
-        for (int r = 0; r < RS; ++r) msum += red[grp * RS + r][lane];
-      __syncthreads();
-      if (rg != 0) continue;
     }
+    /* the sum over layers and query heads, rounded once to fp32 */
+    const float msum = __ull2float_rn(macc) * MASS_UNIT;
+    if (valid && need_mass) p.mass_acc[slot] = 0ull;
     float s = 0.f;
     int pinned = 0;
     if (valid) {
@@ -347,20 +278,11 @@ static int score_grid_cap() {
   return cached[dev];
 }
 
-cudaError_t launch_score(const ScoreParams &p_in, cudaStream_t s) {
-  if (p_in.total_pages == 0) return cudaSuccess;
-  ScoreParams p = p_in;
-  const int ppb = 256 / p.ps;   // pages per block and iteration with one warp per tile
+cudaError_t launch_score(const ScoreParams &p, cudaStream_t s) {
+  if (p.total_pages == 0) return cudaSuccess;
+  const int ppb = 256 / p.ps;   // pages per block and iteration: one warp per tile
   const int cap = p.ps == 16 ? score_grid_cap<16>() : score_grid_cap<32>();
-  /* rows split over up to 8 warps while that still fits one wave and leaves
-   * each warp at least two rows */
-  const long long blocks1 = (p.total_pages + ppb - 1) / ppb;
-  const bool rows_read = p.fold_only || (p.observe && p.mass_pending);
-  p.row_split = 1;
-  while (rows_read && p.row_split < 8 && blocks1 * p.row_split * 2 <= cap && p.rows >= 4 * p.row_split)
-    p.row_split *= 2;
-  const int ppb_rs = ppb / p.row_split;
-  long long blocks = (p.total_pages + ppb_rs - 1) / ppb_rs;
+  long long blocks = (p.total_pages + ppb - 1) / ppb;
   if (blocks > cap) blocks = cap;
   if (p.ps == 16) return launch_pdl(score_kernel<16>, (int)blocks, 256, 0, s, p);
   return launch_pdl(score_kernel<32>, (int)blocks, 256, 0, s, p);

@@ -266,7 +266,7 @@ def test_bit_identical_reruns():
 def test_config2_full_trace_step_is_bit_identical_over_reruns():
     """The full-trace step of the 3B geometry (32 x 1,700 tokens, one split per
     (sequence, layer, KV head), several units per CTA) repeated from one saved
-    state gives bit-identical outputs and mass rows.  A ring stage refilled by
+    state gives bit-identical outputs and step mass.  A ring stage refilled by
     TMA (async proxy) before the consumers' ldmatrix reads of it (generic
     proxy) were fenced showed up here as rare, small differences in one
     item's output (its V rows read after the refill had begun)."""
@@ -306,7 +306,7 @@ def test_config2_full_trace_step_is_bit_identical_over_reruns():
             ref = got
             continue
         assert torch.equal(got[0], ref[0]), f"attention output differs on rerun {rep}"
-        assert torch.equal(got[1], ref[1]), f"mass rows differ on rerun {rep}"
+        assert torch.equal(got[1], ref[1]), f"step mass differs on rerun {rep}"
     assert c.sync() == md.MD_OK
     c.close()
 

@@ -372,7 +372,9 @@ md_status md_calib_fit(const double *mass_sum, const int64_t *count, int n_bucke
  *
  * It runs stage 1 alone -- paged GQA decode attention over every cached
  * token plus each token's attention mass per (layer, KV head) -- over a paged
- * cache the caller already owns, with md_decode_step's kernel and results.
+ * cache the caller already owns, with md_decode_step's kernel (an instance
+ * that writes the masses as rows instead of adding them into one sum per
+ * token) and its arithmetic.
  * The kernel's scratch memory (score rows, split partials, arrival counters,
  * status words) lives in one fixed 24 MiB device array inside the library,
  * which every GPU that loads the library holds until the process exits.

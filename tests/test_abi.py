@@ -57,6 +57,14 @@ def test_workspace_size_is_host_arithmetic(lib):
         assert md.md_workspace_size(_cfg(**bad)) == 0, bad
 
 
+def test_step_mass_headroom_bounds_layers_times_query_heads(lib):
+    """A decode step's mass per token is a u64 with 48 fraction bits, and a
+    token receives at most 1 from each query head of each layer, so the
+    product of layers and query heads must stay below 2^16."""
+    assert md.md_workspace_size(_cfg(num_layers=255, num_q_heads=256, num_kv_heads=32)) > 0
+    assert md.md_workspace_size(_cfg(num_layers=255, num_q_heads=264, num_kv_heads=33)) == 0
+
+
 def test_create_rejects_bad_arguments_before_cuda(lib):
     h = ctypes.c_void_p()
     assert lib.md_create(None, ctypes.byref(h)) == md.MD_ERR_INVALID_ARG
